@@ -1,0 +1,344 @@
+#!/usr/bin/env python
+"""Benchmark of the Ember optimizer step on GB300 (one JSON line on stdout).
+
+A step is one dense Ember step (row/column reduction, state update, apply)
+over one V x D table: by default the large LM head, V = 128256, D = 8192,
+bf16 weights, fp32 gradient and state.  Inputs are resident in HBM when the
+timed region starts; L2 is flushed (a 512 MiB write) between timed steps,
+outside the per-step CUDA events.  `value` is algorithmic bytes per step over
+the mean step time, summed over ranks (independent replicas: the step has no
+cross-GPU exchange on one table held whole by each GPU).
+
+  python bench.py [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+--impl reference times the CPU oracle (plain C, one core) on a bounded row
+sample of the same workload: the paper ships no implementation to compare
+with, so that is the reference arm.
+"""
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "dense_lmhead_v128256_d8192_bf16"
+METRIC = "Ember step GB/s and % of GB300 HBM roofline (dense and sparse), params/sec"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 512 << 20
+
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the apply kernel
+# on the default workload, from the ncu capture summarised in profiles/
+# (None until a capture of the current kernel exists).
+APPLY_TRAFFIC_BYTES = None
+
+
+def wbytes(wl):
+    return 2 if wl.wdtype == "bf16" else 4
+
+
+def step_bytes(wl):
+    """Algorithmic bytes of one dense step: G read twice (every update needs
+    the column statistics of all rows), W read and written once, the V + D
+    state read and written once."""
+    V, D, w = wl.V, wl.D, wbytes(wl)
+    return (8 + 2 * w) * V * D + 8 * (V + D)
+
+
+def kernel_bytes(wl):
+    """Algorithmic bytes per launch of each kernel of the dense step."""
+    V, D, w = wl.V, wl.D, wbytes(wl)
+    return {"reduce": 4 * V * D + 8 * V, "state": 8 * D, "apply": (4 + 2 * w) * V * D + 4 * (V + D)}
+
+
+def measured_hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu_index = gpu_index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.out = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.out, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.out.close()
+
+    def summary(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                p = [x.strip() for x in line.split(",")]
+                if len(p) >= 9 and p[1].replace(".", "").isdigit():
+                    rows.append(p)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"], "samples": 0}
+        sm = sorted(float(p[1]) for p in rows)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({n for p in rows for n, v in zip(names, p[5:9]) if v.lower() == "active"})
+        return {"sm_mhz": sm[len(sm) // 2], "sm_max_mhz": float(rows[0][2]), "reasons": reasons,
+                "samples": len(rows), "power_w_max": max(float(p[3]) for p in rows)}
+
+
+def oracle_sample(wl, rows, seed=0):
+    """The oracle's dense step on the first `rows` rows of the workload (a
+    rows x D table with the workload's generator); returns seconds."""
+    import numpy as np
+    import torch
+    import oracle
+    from paper_2607_01455_gb300 import synth
+    sub = synth.Workload(wl.name + "_sample", rows, wl.D, wl.wdtype, 1,
+                         zero_frac=wl.zero_frac, heavy_frac=wl.heavy_frac)
+    W = synth.init_weights(sub, seed, "cpu")
+    W = W.view(torch.int16).numpy().view(np.uint16).copy() if wl.wdtype == "bf16" else W.numpy().copy()
+    G = synth.dense_grad(sub, seed, 1, "cpu").numpy()
+    r = np.zeros(rows, np.float32)
+    c = np.zeros(wl.D, np.float32)
+    t0 = time.perf_counter()
+    oracle.step_dense(W, G, r, c, wl.lr, 1)
+    return time.perf_counter() - t0
+
+
+def sample_rows_for(wl, seconds):
+    """Rows of a sample whose oracle step takes about `seconds`."""
+    probe = 64
+    dt = oracle_sample(wl, probe)
+    return int(max(16, min(wl.V, probe * seconds / max(dt, 1e-6))))
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("gloo")
+    return world, rank, local
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+def allreduce_max(world, x):
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_reference(args, world, rank):
+    from paper_2607_01455_gb300 import synth
+    wl = synth.WORKLOADS[args.workload]
+    if rank != 0:
+        return 0
+    budget = 90.0  # seconds for the whole warm-up + timed run
+    rows = sample_rows_for(wl, budget / (args.steps + args.warmup))
+    sub_bytes = step_bytes(synth.Workload("s", rows, wl.D, wl.wdtype, 1))
+    for _ in range(args.warmup):
+        oracle_sample(wl, rows)
+    times = [oracle_sample(wl, rows) for _ in range(args.steps)]
+    sec = sum(times) / len(times)
+    gbs = sub_bytes / sec / 1e9
+    sample = f"oracle dense step on the first {rows} of {wl.V} rows (D={wl.D}, {wl.wdtype} W), one thread"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": wl.name, "V": wl.V, "D": wl.D,
+                                        "w_dtype": wl.wdtype, "sample_rows": rows},
+        "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def run_ours(args, world, rank, local):
+    import torch
+    from paper_2607_01455_gb300 import synth
+    from paper_2607_01455_gb300.ember import Ember
+
+    wl = synth.WORKLOADS[args.workload]
+    if wl.kind != "dense":
+        raise SystemExit("bench.py times the dense workloads")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream(dev)
+
+    W = synth.init_weights(wl, rank, dev)
+    G = synth.dense_grad(wl, rank, 1, dev)
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
+
+    def one_step(t, ev):
+        emb.trace(ev)
+        emb.step_dense(W, G, wl.lr, t)
+
+    warm_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    t = 0
+    for _ in range(args.warmup):
+        t += 1
+        flush.zero_()
+        one_step(t, warm_ev)
+    torch.cuda.synchronize()
+
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    with ClockSampler(local) as clocks:
+        for k in range(args.steps):
+            t += 1
+            flush.zero_()
+            one_step(t, events[k])
+        torch.cuda.synchronize()
+        barrier(world)
+    wall = time.perf_counter() - wall0
+    emb.trace([])
+    status = emb.device_status()
+    if status != 0:
+        raise SystemExit(f"device status {status} after the timed steps")
+
+    per = {"reduce": [], "state": [], "apply": [], "step": []}
+    for ev in events:
+        per["reduce"].append(ev[0].elapsed_time(ev[1]))
+        per["state"].append(ev[1].elapsed_time(ev[2]))
+        per["apply"].append(ev[2].elapsed_time(ev[3]))
+        per["step"].append(ev[0].elapsed_time(ev[3]))
+    mean = {k: sum(v) / len(v) for k, v in per.items()}
+    ms = allreduce_max(world, mean["step"])
+
+    B = step_bytes(wl)
+    value = world * B / (ms * 1e-3) / 1e9
+    peak, peak_kind = measured_hbm_peak()
+    kb = kernel_bytes(wl)
+    kern = {k: {"ms": mean[k], "gbs": kb[k] / (mean[k] * 1e-3) / 1e9} for k in ("reduce", "state", "apply")}
+    dom = "apply"
+    roofline = {
+        "bound": "hbm", "kernel": "k_apply_dense", "achieved": kern[dom]["gbs"], "peak": peak,
+        "unit": "GB/s", "frac": kern[dom]["gbs"] / peak, "peak_kind": peak_kind,
+        "traffic": APPLY_TRAFFIC_BYTES,
+        "algorithmic_bytes_per_launch": kb[dom],
+    }
+
+    # end to end through the C ABI: pinned host gradient in, updated weights out
+    e2e = None
+    if not args.no_e2e:
+        n_e2e = max(1, min(args.steps, 5))
+        Gh = G.cpu().pin_memory()
+        Wh = torch.empty(W.shape, dtype=W.dtype, pin_memory=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        G2 = torch.empty_like(G)
+        ts = []
+        for _ in range(n_e2e):
+            t += 1
+            flush.zero_()
+            e0.record(stream)
+            G2.copy_(Gh, non_blocking=True)
+            emb.step_dense(W, G2, wl.lr, t)
+            Wh.copy_(W, non_blocking=True)
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
+        ms_e2e = allreduce_max(world, sum(ts) / len(ts))
+        e2e = {"value": world * B / (ms_e2e * 1e-3) / 1e9, "unit": "GB/s",
+               "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": W.numel() * W.element_size(),
+               "ms_per_step": ms_e2e, "steps": n_e2e}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        rows = sample_rows_for(wl, 5.0)
+        secs = [oracle_sample(wl, rows) for _ in range(3)]
+        sub = synth.Workload("s", rows, wl.D, wl.wdtype, 1)
+        sec = sum(secs) / len(secs)
+        cpu = {"value": step_bytes(sub) / sec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+               "sample": f"3 oracle dense steps on the first {rows} of {wl.V} rows (D={wl.D}), one thread",
+               "ms_per_step": sec * 1e3}
+
+    line = {
+        "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "w_dtype": wl.wdtype, "g_dtype": "f32",
+                   "state_dtype": "f32", "l2": "flushed between steps (512 MiB write, outside the events)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": roofline,
+        "cpu_baseline": cpu,
+        "e2e": e2e,
+        "gpu_launches": 3 * args.steps,
+        "clocks": clocks.summary(),
+        "params_per_s": world * wl.V * wl.D / (ms * 1e-3),
+        "frac_of_nominal_8TBs": value / world / NOMINAL_HBM_GBS,
+        "frac_of_measured_hbm": value / world / peak,
+        "kernels": kern,
+        "wall_s_timed_region": wall,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    world, rank, local = dist_setup()
+    if args.impl == "reference":
+        rc = run_reference(args, world, rank)
+    else:
+        rc = run_ours(args, world, rank, local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+    return rc
+
+
+if __name__ == "__main__":
+    sys.exit(main())

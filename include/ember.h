@@ -1,0 +1,175 @@
+/*
+ * ember.h -- C ABI of the Ember optimizer step for V x D token tables
+ * (embedding tables and LM heads), GB300 (sm_103a) CUDA implementation.
+ *
+ * Ember is Algorithm 1 of "Token Geometry" (arXiv 2607.01455, Section 2.1).
+ * For a table W (V rows = tokens, D columns = features) and its gradient g
+ * at step t it keeps only two fp32 vectors, r (V) and c (D), and does:
+ *
+ *   r <- beta2 r + (1-beta2) mean_j g_ij^2          (row second moment)
+ *   c <- beta2 c + (1-beta2) mean_i g_ij^2          (column second moment)
+ *   rhat = r / (1-beta2^t),  chat = c / (1-beta2^t) (bias correction)
+ *   s = sqrt(mean_i rhat_i * mean_j chat_j)         (geometric-mean normaliser)
+ *   W_ij <- W_ij - lr * g_ij / (sqrt(rhat_i chat_j / s) + eps)
+ *
+ * The V x D preconditioner rhat chat^T / s is never stored: it is applied as
+ * a per-row and a per-column scaling (Section 2.3, "The preconditioner is
+ * never stored").  The sparse step (Section 2.2) takes the token ids of a
+ * batch and one gradient row per occurrence; it equals the dense step on the
+ * V x D gradient whose row u is the sum of the rows of every occurrence of u.
+ *
+ * Conventions shared by every entry point:
+ *   - Device pointers are CUDA device (or managed) addresses on the current
+ *     device; every array is row-major and contiguous.  The library never
+ *     allocates or frees device memory: W, G, ids, rows, the state and the
+ *     workspace belong to the caller.
+ *   - "stream" is a cudaStream_t passed as void* (NULL = the legacy default
+ *     stream).  Steps are asynchronous on that stream.  Errors the host can
+ *     see are returned at once and nothing is launched; errors only the GPU
+ *     can see (an id outside [0, V), a bounded wait that gave up) set a
+ *     sticky flag in the workspace that ember_get_device_status() reads.
+ *   - A handle is not thread-safe; use one handle per table and do not run
+ *     two steps of one handle concurrently on different streams (they share
+ *     the workspace).
+ *   - Results are deterministic: the same inputs give bit-identical W and
+ *     state on every run.  No floating-point atomics are used; every sum is
+ *     taken in a fixed order (Section 2.3, "deterministic reduction with no
+ *     atomic adds").
+ */
+#ifndef EMBER_H
+#define EMBER_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define EMBER_ABI_VERSION 1
+
+typedef enum {
+    EMBER_OK = 0,
+    EMBER_ERR_INVALID_ARG = 1,     /* null pointer, bad size, t < 1, beta2 outside [0,1), ... */
+    EMBER_ERR_ALIGNMENT = 2,       /* a pointer is not aligned to its element size */
+    EMBER_ERR_DTYPE = 3,           /* unknown weight or id type */
+    EMBER_ERR_WORKSPACE = 4,       /* no workspace bound, or too small for this call */
+    EMBER_ERR_CUDA = 5,            /* a CUDA runtime call or a kernel launch failed */
+    EMBER_ERR_ID_OUT_OF_RANGE = 6, /* device flag: a token id was outside [0, V) and was skipped */
+    EMBER_ERR_TIMEOUT = 7,         /* device flag: a bounded wait inside a kernel gave up */
+    EMBER_ERR_UNSUPPORTED = 8      /* the GPU is not sm_103 or the size is beyond a stated limit */
+} ember_status;
+
+typedef enum { EMBER_F32 = 0, EMBER_BF16 = 1 } ember_wdtype;  /* storage type of W */
+typedef enum { EMBER_I32 = 0, EMBER_I64 = 1 } ember_idtype;   /* storage type of token ids */
+
+/* Preconditioner.  FULL is Algorithm 1.  ROW (vtil_ij = rhat_i, a V-float
+ * state in use) and COL (vtil_ij = chat_j) are the "row-only" and "col-only"
+ * rows of the ablation table in Section 2.1; both keep the same V + D state
+ * layout so that a handle can switch between them. */
+typedef enum {
+    EMBER_VARIANT_FULL = 0,
+    EMBER_VARIANT_ROW = 1,
+    EMBER_VARIANT_COL = 2
+} ember_variant;
+
+typedef struct {
+    double beta2;        /* second-moment decay, in [0, 1).  Default 0.999 (Algorithm 1). */
+    double eps;          /* added to sqrt(vtil), >= 0.  Default 1e-8 (Algorithm 1). */
+    int maximize;        /* 0 (default): W -= lr u, descending a loss whose gradient is G.
+                            1: W += lr u, ascending a reward, as Algorithm 1 is printed. */
+    int bias_correction; /* 1 (default): divide by 1 - beta2^t.  0: the ablation of the
+                            appendix "Ablations" (rhat = r, chat = c). */
+    int variant;         /* ember_variant; default EMBER_VARIANT_FULL */
+} ember_hparams;
+
+typedef struct ember_handle ember_handle;
+
+/* Fill *hp with the defaults of Algorithm 1: beta2 = 0.999, eps = 1e-8,
+ * descent, bias correction on, full preconditioner. */
+void ember_hparams_default(ember_hparams *hp);
+
+/* Create a host-side handle for one V x D table whose weights are stored as
+ * wdtype.  hp == NULL takes the defaults.  Validates V >= 1, D >= 1,
+ * V * D < 2^62, 0 <= beta2 < 1, eps >= 0 (finite) and the enums.  Touches no
+ * GPU.  On success *out owns a handle to free with ember_destroy(). */
+ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp,
+                          ember_wdtype wdtype, ember_handle **out);
+
+/* Free the host handle (never device memory).  NULL is ignored. */
+void ember_destroy(ember_handle *h);
+
+/* Number of fp32 values of optimizer state: exactly V + D (Algorithm 1
+ * keeps r in R^V and c in R^D).  The caller's state buffer holds r in
+ * [0, V) followed by c in [V, V + D).  A new table starts from all zeros
+ * (Algorithm 1 initialises r_0 = 0 and c_0 = 0). */
+size_t ember_state_numel(const ember_handle *h);
+
+/* Bytes of device workspace the steps of this handle need when sparse steps
+ * carry at most max_sparse_N ids (0 if only dense steps are used).  Returns
+ * 0 for a NULL handle or a negative max_sparse_N.  The workspace holds
+ * per-block partial sums, the sort buffers of the sparse step, the summed
+ * gradient rows of the sparse step (up to max_sparse_N x D fp32) and a few
+ * scalars; it is not optimizer state and need not persist between steps,
+ * but the caller must not touch it while a step is in flight. */
+size_t ember_workspace_bytes(const ember_handle *h, int64_t max_sparse_N);
+
+/* Give the handle its device workspace (256-byte aligned, at least
+ * ember_workspace_bytes(h, max_sparse_N) bytes) and clear the sticky device
+ * flag with a memset on `stream`.  Rebinding replaces the previous
+ * workspace. */
+ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes,
+                                  int64_t max_sparse_N, void *stream);
+
+/* One dense Ember step (Algorithm 1) at step number t >= 1.
+ *   W:     V x D, wdtype, updated in place.
+ *   G:     V x D fp32 gradient of the loss (of the reward when maximize = 1).
+ *   state: V + D fp32 (r then c), updated in place.
+ *   lr:    step size alpha, applied in fp32 (any finite value).
+ * W and G must be 4-byte (bf16 W: 2-byte) aligned; with D % 4 == 0 and
+ * 16-byte aligned W, G and state the vectorised kernels run, otherwise a
+ * scalar path gives the same results more slowly. */
+ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *state,
+                              float lr, int64_t t, void *stream);
+
+/* One sparse Ember step (Section 2.2) at step number t >= 1.
+ *   ids:   N token ids of type idtype (duplicates allowed, any order).
+ *   rows:  N x D fp32, row k is the gradient contribution of occurrence k
+ *          (any 1/batch scaling already applied by the caller).
+ *   N:     0 <= N <= the max_sparse_N the workspace was bound for.
+ * Equals ember_step_dense on the V x D gradient whose row u is the sum of
+ * rows[k] over the k with ids[k] == u, summed in increasing k: every row of
+ * r decays by beta2, the column statistics divide by V, and rows of W whose
+ * id does not occur are left bit-identical.  An id outside [0, V) is
+ * skipped and sets EMBER_ERR_ID_OUT_OF_RANGE in the device flag. */
+ember_status ember_step_sparse(ember_handle *h, void *W, const void *ids,
+                               ember_idtype idtype, int64_t N, const float *rows,
+                               float *state, float lr, int64_t t, void *stream);
+
+/* Synchronise `stream`, return the sticky device flag of this handle's
+ * workspace (EMBER_OK if no device error happened since the last call) and
+ * clear it. */
+ember_status ember_get_device_status(ember_handle *h, void *stream);
+
+/* Kernel-boundary tracing.  events[k] are cudaEvent_t handles owned by the
+ * caller (created on the current device); n of them, at most 16.  While set,
+ * every step records events[0] on its stream before its first kernel and
+ * events[k] after its k-th kernel, so cudaEventElapsedTime(events[k-1],
+ * events[k]) is the device time of kernel k.  The dense step launches 3
+ * kernels (reduce, state, apply), so it records events[0..3]; the sparse
+ * step records one event per kernel it launches, up to n - 1.  Pass
+ * events = NULL or n = 0 to stop tracing.  The events are not recorded
+ * when n is too small for a step; nothing else changes. */
+ember_status ember_set_trace_events(ember_handle *h, void *const *events, int n);
+
+/* Static description of a status code. */
+const char *ember_status_string(ember_status s);
+
+/* EMBER_ABI_VERSION of the compiled library. */
+int ember_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EMBER_H */

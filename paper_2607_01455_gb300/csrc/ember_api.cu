@@ -1,0 +1,249 @@
+// Host side of the C ABI declared in include/ember.h: argument checks,
+// workspace layout and kernel dispatch.  Every check runs before anything is
+// launched, so a rejected call leaves the GPU untouched.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#include "ember_internal.h"
+
+namespace ember {
+
+static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
+{
+    (void)V;
+    Layout L{};
+    size_t off = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = off;
+        off = align_up(off + (bytes ? bytes : 1), 256);
+        return at;
+    };
+    const size_t nstate = (size_t)((D + kStateCols - 1) / kStateCols);
+    L.scalars = take(sizeof(DevScalars));
+    L.rsum_part = take(sizeof(double) * kGridCtas);
+    L.csum_part = take(sizeof(double) * nstate);
+    L.colpart = take(sizeof(float) * (size_t)kGridCtas * (size_t)D);
+    if (max_sparse_N > 0) {
+        const size_t N = (size_t)max_sparse_N;
+        L.sp_keys = take(sizeof(uint64_t) * N);
+        L.sp_sorted = take(sizeof(uint64_t) * N);
+        L.sp_head = take(sizeof(int32_t) * (N + 1));
+        L.sp_uniq = take(sizeof(int32_t) * N);
+        L.sp_segoff = take(sizeof(int32_t) * (N + 1));
+        L.sp_tilecnt = take(sizeof(int32_t) * (N + 2));
+        L.sp_rows = take(sizeof(float) * N * (size_t)D);
+    }
+    L.total = off;
+    return L;
+}
+
+}  // namespace ember
+
+using namespace ember;
+
+static bool is_aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+static bool hparams_ok(const ember_hparams &hp)
+{
+    return hp.beta2 >= 0.0 && hp.beta2 < 1.0 && isfinite(hp.eps) && hp.eps >= 0.0 &&
+           (hp.maximize == 0 || hp.maximize == 1) &&
+           (hp.bias_correction == 0 || hp.bias_correction == 1) &&
+           hp.variant >= EMBER_VARIANT_FULL && hp.variant <= EMBER_VARIANT_COL;
+}
+
+extern "C" {
+
+void ember_hparams_default(ember_hparams *hp)
+{
+    if (!hp)
+        return;
+    hp->beta2 = 0.999;
+    hp->eps = 1e-8;
+    hp->maximize = 0;
+    hp->bias_correction = 1;
+    hp->variant = EMBER_VARIANT_FULL;
+}
+
+ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp, ember_wdtype wdtype,
+                          ember_handle **out)
+{
+    if (!out)
+        return EMBER_ERR_INVALID_ARG;
+    *out = nullptr;
+    if (V < 1 || D < 1 || V > (int64_t(1) << 62) / D)
+        return EMBER_ERR_INVALID_ARG;
+    if (D > INT32_MAX || V > INT32_MAX)
+        return EMBER_ERR_UNSUPPORTED;
+    if (wdtype != EMBER_F32 && wdtype != EMBER_BF16)
+        return EMBER_ERR_DTYPE;
+    ember_hparams h;
+    if (hp)
+        h = *hp;
+    else
+        ember_hparams_default(&h);
+    if (!hparams_ok(h))
+        return EMBER_ERR_INVALID_ARG;
+    ColMap m;
+    if (!choose_colmap(D, true, &m))  // wider rows than one CTA holds
+        return EMBER_ERR_UNSUPPORTED;
+    ember_handle *e = (ember_handle *)calloc(1, sizeof(ember_handle));
+    if (!e)
+        return EMBER_ERR_INVALID_ARG;
+    e->V = V;
+    e->D = D;
+    e->hp = h;
+    e->wdtype = wdtype;
+    *out = e;
+    return EMBER_OK;
+}
+
+void ember_destroy(ember_handle *h) { free(h); }
+
+size_t ember_state_numel(const ember_handle *h)
+{
+    return h ? (size_t)(h->V + h->D) : 0;
+}
+
+size_t ember_workspace_bytes(const ember_handle *h, int64_t max_sparse_N)
+{
+    if (!h || max_sparse_N < 0 || max_sparse_N > INT32_MAX / 2)
+        return 0;
+    return make_layout(h->V, h->D, max_sparse_N).total;
+}
+
+ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes,
+                                  int64_t max_sparse_N, void *stream)
+{
+    if (!h || !workspace || max_sparse_N < 0 || max_sparse_N > INT32_MAX / 2)
+        return EMBER_ERR_INVALID_ARG;
+    if (!is_aligned(workspace, 256))
+        return EMBER_ERR_ALIGNMENT;
+    const Layout L = make_layout(h->V, h->D, max_sparse_N);
+    if (bytes < L.total)
+        return EMBER_ERR_WORKSPACE;
+    int dev = 0;
+    cudaDeviceProp prop;
+    if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess)
+        return EMBER_ERR_CUDA;
+    if (prop.major != 10 || prop.minor != 3)
+        return EMBER_ERR_UNSUPPORTED;
+    if (cudaMemsetAsync((unsigned char *)workspace + L.scalars, 0, sizeof(DevScalars),
+                        (cudaStream_t)stream) != cudaSuccess)
+        return EMBER_ERR_CUDA;
+    h->ws = (unsigned char *)workspace;
+    h->ws_bytes = bytes;
+    h->ws_max_N = max_sparse_N;
+    return EMBER_OK;
+}
+
+ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *state, float lr,
+                              int64_t t, void *stream)
+{
+    if (!h || !W || !G || !state)
+        return EMBER_ERR_INVALID_ARG;
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    if (!is_aligned(W, wsz) || !is_aligned(G, 4) || !is_aligned(state, 4))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+
+    DenseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.wbf16 = h->wdtype == EMBER_BF16;
+    a.W = W;
+    a.G = G;
+    a.r = state;
+    a.c = state + h->V;
+    a.beta2 = h->hp.beta2;
+    a.one_minus_beta2 = 1.0 - h->hp.beta2;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.eps = (float)h->hp.eps;
+    a.variant = h->hp.variant;
+    a.ws = h->ws;
+    a.lay = make_layout(h->V, h->D, h->ws_max_N);
+    a.stream = (cudaStream_t)stream;
+    a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && is_aligned(G, 16);
+    if (!choose_colmap(h->D, vec4, &a.map))
+        return EMBER_ERR_UNSUPPORTED;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+ember_status ember_step_sparse(ember_handle *h, void *W, const void *ids, ember_idtype idtype,
+                               int64_t N, const float *rows, float *state, float lr, int64_t t,
+                               void *stream)
+{
+    (void)stream;
+    if (!h || !W || !state || N < 0 || (N > 0 && (!ids || !rows)))
+        return EMBER_ERR_INVALID_ARG;
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    if (idtype != EMBER_I32 && idtype != EMBER_I64)
+        return EMBER_ERR_DTYPE;
+    return EMBER_ERR_UNSUPPORTED;
+}
+
+ember_status ember_get_device_status(ember_handle *h, void *stream)
+{
+    if (!h)
+        return EMBER_ERR_INVALID_ARG;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    const Layout L = make_layout(h->V, h->D, h->ws_max_N);
+    DevScalars *sc = reinterpret_cast<DevScalars *>(h->ws + L.scalars);
+    unsigned flags = 0;
+    if (cudaMemcpyAsync(&flags, &sc->flags, sizeof flags, cudaMemcpyDeviceToHost, s) != cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return EMBER_ERR_CUDA;
+    if (flags && (cudaMemsetAsync(&sc->flags, 0, sizeof(unsigned), s) != cudaSuccess ||
+                  cudaStreamSynchronize(s) != cudaSuccess))
+        return EMBER_ERR_CUDA;
+    if (flags & kFlagTimeout)
+        return EMBER_ERR_TIMEOUT;
+    if (flags & kFlagIdRange)
+        return EMBER_ERR_ID_OUT_OF_RANGE;
+    return EMBER_OK;
+}
+
+ember_status ember_set_trace_events(ember_handle *h, void *const *events, int n)
+{
+    if (!h || n < 0 || n > kMaxTraceEvents || (n > 0 && !events))
+        return EMBER_ERR_INVALID_ARG;
+    for (int k = 0; k < n; ++k)
+        if (!events[k])
+            return EMBER_ERR_INVALID_ARG;
+    h->n_trace = events ? n : 0;
+    for (int k = 0; k < h->n_trace; ++k)
+        h->trace[k] = (cudaEvent_t)events[k];
+    return EMBER_OK;
+}
+
+const char *ember_status_string(ember_status s)
+{
+    switch (s) {
+    case EMBER_OK: return "ok";
+    case EMBER_ERR_INVALID_ARG: return "invalid argument";
+    case EMBER_ERR_ALIGNMENT: return "misaligned pointer";
+    case EMBER_ERR_DTYPE: return "unknown dtype";
+    case EMBER_ERR_WORKSPACE: return "workspace missing or too small";
+    case EMBER_ERR_CUDA: return "CUDA error";
+    case EMBER_ERR_ID_OUT_OF_RANGE: return "token id outside [0, V) skipped";
+    case EMBER_ERR_TIMEOUT: return "bounded device wait gave up";
+    case EMBER_ERR_UNSUPPORTED: return "unsupported device or size";
+    }
+    return "unknown status";
+}
+
+int ember_abi_version(void) { return EMBER_ABI_VERSION; }
+
+}  // extern "C"

@@ -1,0 +1,512 @@
+// Dense Ember step (Algorithm 1 of "Token Geometry", arXiv 2607.01455,
+// Section 2.1) for sm_103a.
+//
+// The step needs two passes over the fp32 gradient G: the update of any
+// element needs chat_j and s, which depend on every row of G (Section 2.3:
+// "The statistics r and c are sums of g^2").  The passes are:
+//
+//   reduce  (k_reduce_dense)  one read of G.  Per row: sum_j g^2, the row EMA
+//           r_i <- beta2 r_i + (1-beta2) mean_j g^2 (Algorithm 1's row second
+//           moment), written once.  Per CTA: column sums of g^2 over its rows
+//           and the sum of its new r values, written to the workspace.
+//   state   (k_state_dense)   O(D * CTAs) work: column sums in a fixed order,
+//           the column EMA c_j <- beta2 c_j + (1-beta2) mean_i g^2, then the
+//           last CTA forms mean(rhat), mean(chat) and s = sqrt(mean rhat *
+//           mean chat) (the geometric-mean normaliser).
+//   apply   (k_apply_dense)   reads G and W, writes W:
+//           W_ij <- W_ij - lr g_ij / (sqrt(rhat_i) sqrt(chat_j / s) + eps),
+//           the factored preconditioner applied as a row scale times a
+//           column scale, never stored (Section 2.3).
+//
+// Bandwidth: 4VD bytes (reduce) + 4VD + 2 w VD bytes (apply), w = bytes per
+// weight.  The apply pass walks each CTA's rows in the reverse order of the
+// reduce pass, so the rows read last by the reduce pass -- still in L2 --
+// are the first ones it needs.
+//
+// Determinism: no floating-point atomics.  Every CTA owns a fixed row range
+// (a function of V only), every in-CTA sum has a fixed shape, and the
+// cross-CTA sums run in CTA order, so W and the state are bit-identical
+// from run to run (Section 2.3: "bitwise identical").
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "ember_internal.h"
+
+namespace ember {
+namespace {
+
+template <int VEC> struct Vec;
+template <> struct Vec<4> { using F = float4; };
+template <> struct Vec<1> { using F = float; };
+
+__device__ __forceinline__ float comp(const float4 &v, int e)
+{
+    return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
+}
+__device__ __forceinline__ float comp(const float &v, int) { return v; }
+__device__ __forceinline__ void set_comp(float4 &v, int e, float x)
+{
+    if (e == 0) v.x = x; else if (e == 1) v.y = x; else if (e == 2) v.z = x; else v.w = x;
+}
+__device__ __forceinline__ void set_comp(float &v, int, float x) { v = x; }
+
+template <int VEC>
+__device__ __forceinline__ typename Vec<VEC>::F load_g(const float *p)
+{
+    if constexpr (VEC == 4)
+        return __ldg(reinterpret_cast<const float4 *>(p));
+    else
+        return __ldg(p);
+}
+
+template <int VEC>
+__device__ __forceinline__ typename Vec<VEC>::F zero_vec()
+{
+    if constexpr (VEC == 4)
+        return make_float4(0.f, 0.f, 0.f, 0.f);
+    else
+        return 0.f;
+}
+
+// Sum R per-lane values over the 32 lanes of a warp, "transposed": each
+// halving step trades half of the values with a partner lane, so the R
+// totals cost R-1 + log2(32/R) shuffles instead of 5R.  On return v[0] of
+// lane l is the warp total of value index `row` (lanes whose low
+// log2(32/R) bits differ hold the same total).  The addition tree is fixed,
+// so the result is the same on every run.
+template <int R>
+__device__ __forceinline__ float warp_sum_transposed(float (&v)[R], int lane, int &row)
+{
+    static_assert(R >= 1 && R <= 32 && (R & (R - 1)) == 0, "R must be a power of two <= 32");
+    constexpr int kLog = (R >= 32) ? 5 : (R >= 16) ? 4 : (R >= 8) ? 3 : (R >= 4) ? 2 : (R >= 2) ? 1 : 0;
+    row = 0;
+#pragma unroll
+    for (int s = 0; s < kLog; ++s) {
+        const int o = 16 >> s;
+        const int h = R >> (s + 1);
+        const bool hi = (lane & o) != 0;
+#pragma unroll
+        for (int m = 0; m < h; ++m) {
+            const float send = hi ? v[m] : v[m + h];
+            const float keep = hi ? v[m + h] : v[m];
+            v[m] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+        if (hi)
+            row += h;
+    }
+#pragma unroll
+    for (int o = 16 >> kLog; o >= 1; o >>= 1)
+        v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
+    return v[0];
+}
+
+// Pass 1: one read of G.  Template: VEC columns per access, CPT accesses per
+// thread per row, R rows per row group per iteration.
+template <int VEC, int CPT, int R>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
+               float *__restrict__ colpart, double *__restrict__ rsum_part,
+               int64_t V, int D, int tpr, double beta2, double one_minus_beta2)
+{
+    using F = typename Vec<VEC>::F;
+    constexpr int kWarps = kThreads / 32;
+    const int DV = D / VEC;
+    const int tid = threadIdx.x;
+    const int lane = tid & 31;
+    const int warp = tid >> 5;
+    const int rg = kThreads / tpr;           // row groups
+    const int g = tid / tpr;                 // this thread's row group
+    const int l = tid - g * tpr;             // position within the row
+    const int wpg = tpr >> 5;                // warps per row group
+    const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
+    const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+
+    __shared__ float red[2][kWarps][R];
+    __shared__ double rsum_sh[kThreads];
+
+    float acc[CPT][VEC];
+#pragma unroll
+    for (int c = 0; c < CPT; ++c)
+#pragma unroll
+        for (int e = 0; e < VEC; ++e)
+            acc[c][e] = 0.f;
+    double rsum = 0.0;
+
+    int buf = 0;
+    for (int64_t base = row0; base < row1; base += (int64_t)rg * R, buf ^= 1) {
+        F v[R][CPT];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col = l + c * tpr;
+                v[k][c] = (i < row1 && col < DV) ? load_g<VEC>(G + i * D + (int64_t)col * VEC)
+                                                 : zero_vec<VEC>();
+            }
+        }
+        // squares and per-row partial sums
+        float rp[R];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            float s = 0.f;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c)
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const float x = comp(v[k][c], e);
+                    const float x2 = x * x;
+                    set_comp(v[k][c], e, x2);
+                    s += x2;
+                }
+            rp[k] = s;
+        }
+        // column sums: pairwise over the R rows of this iteration, then into acc
+#pragma unroll
+        for (int w = R / 2; w >= 1; w >>= 1)
+#pragma unroll
+            for (int k = 0; k < w; ++k)
+#pragma unroll
+                for (int c = 0; c < CPT; ++c)
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e)
+                        set_comp(v[k][c], e, comp(v[k][c], e) + comp(v[k + w][c], e));
+#pragma unroll
+        for (int c = 0; c < CPT; ++c)
+#pragma unroll
+            for (int e = 0; e < VEC; ++e)
+                acc[c][e] += comp(v[0][c], e);
+
+        // row sums: within the warp, then across the warps of the row group
+        int row_in_warp;
+        const float tot = warp_sum_transposed<R>(rp, lane, row_in_warp);
+        if ((lane & (32 / R - 1)) == 0)
+            red[buf][warp][row_in_warp] = tot;
+        __syncthreads();
+        if (l < R) {
+            const int64_t i = base + (int64_t)g * R + l;
+            if (i < row1) {
+                float sum = 0.f;
+                for (int q = 0; q < wpg; ++q)
+                    sum += red[buf][g * wpg + q][l];
+                const double mean_row = (double)sum / (double)D;
+                const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
+                r[i] = rn;
+                rsum += (double)rn;
+            }
+        }
+        // the next iteration writes the other buffer; the one after that
+        // writes this buffer again only after the next __syncthreads().
+    }
+
+    // column partial of this CTA: row groups combined in order 0 .. rg-1
+    float *out = colpart + (int64_t)blockIdx.x * D;
+    if (rg == 1) {
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+            const int col = l + c * tpr;
+            if (col < DV)
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    out[col * VEC + e] = acc[c][e];
+        }
+    } else {
+        extern __shared__ float colsh[];  // D floats
+        for (int q = 0; q < rg; ++q) {
+            if (g == q) {
+#pragma unroll
+                for (int c = 0; c < CPT; ++c) {
+                    const int col = l + c * tpr;
+                    if (col < DV)
+#pragma unroll
+                        for (int e = 0; e < VEC; ++e)
+                            colsh[col * VEC + e] = (q == 0) ? acc[c][e] : colsh[col * VEC + e] + acc[c][e];
+                }
+            }
+            __syncthreads();
+        }
+        for (int j = tid; j < D; j += kThreads)
+            out[j] = colsh[j];
+    }
+
+    // sum of the new r values of this CTA, threads in order
+    rsum_sh[tid] = rsum;
+    __syncthreads();
+    if (tid == 0) {
+        double s = 0.0;
+        for (int q = 0; q < kThreads; ++q)
+            s += rsum_sh[q];
+        rsum_part[blockIdx.x] = s;
+    }
+}
+
+// Pass 2: column EMA and the normaliser.  CTA x owns columns
+// [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in order.
+__global__ void __launch_bounds__(kStateThreads)
+k_state_dense(const float *__restrict__ colpart, int nparts, const double *__restrict__ rsum_part,
+              float *__restrict__ c, double *__restrict__ csum_part, DevScalars *sc,
+              int64_t V, int D, double beta2, double one_minus_beta2, double inv_bc)
+{
+    constexpr int kW = kStateThreads / 32;
+    const int lane = threadIdx.x & 31;
+    const int w = threadIdx.x >> 5;
+    const int j = blockIdx.x * kStateCols + lane;
+    __shared__ double part[kW][32];
+    __shared__ bool am_last;
+
+    double acc = 0.0;
+    if (j < D)
+        for (int b = w; b < nparts; b += kW)
+            acc += (double)colpart[(int64_t)b * D + j];
+    part[w][lane] = acc;
+    __syncthreads();
+    if (w == 0) {
+        double tot = 0.0;
+#pragma unroll
+        for (int q = 0; q < kW; ++q)
+            tot += part[q][lane];
+        double cn = 0.0;
+        if (j < D) {
+            const double mean_col = tot / (double)V;
+            const float cnew = (float)(beta2 * (double)c[j] + one_minus_beta2 * mean_col);
+            c[j] = cnew;
+            cn = (double)cnew;
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1)
+            cn += __shfl_xor_sync(0xffffffffu, cn, o);
+        if (lane == 0)
+            csum_part[blockIdx.x] = cn;
+    }
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const unsigned t = atomicAdd(&sc->ticket, 1u);
+        am_last = (t == gridDim.x - 1);
+    }
+    __syncthreads();
+    if (am_last && threadIdx.x == 0) {
+        __threadfence();
+        const volatile double *cp = csum_part;
+        double csum = 0.0;
+        for (int b = 0; b < (int)gridDim.x; ++b)
+            csum += cp[b];
+        double rsum = 0.0;
+        for (int b = 0; b < nparts; ++b)
+            rsum += rsum_part[b];
+        const double rbar = rsum * inv_bc / (double)V;
+        const double cbar = csum * inv_bc / (double)D;
+        const double s = sqrt(rbar * cbar);
+        sc->s = s;
+        sc->rbar = rbar;
+        sc->cbar = cbar;
+        sc->inv_s = (s > 0.0) ? (float)(1.0 / s) : 0.f;
+        sc->ticket = 0u;
+    }
+}
+
+__device__ __forceinline__ float bf16_lo(unsigned u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf16_hi(unsigned u) { return __uint_as_float(u & 0xFFFF0000u); }
+__device__ __forceinline__ unsigned short f2bf(float x)
+{
+    return __bfloat16_as_ushort(__float2bfloat16_rn(x));
+}
+
+// Raw weight vectors: kept packed between the load and the update.
+template <bool BF16, int VEC> struct WRaw;
+template <> struct WRaw<true, 4> { using T = uint2; };
+template <> struct WRaw<true, 1> { using T = unsigned short; };
+template <> struct WRaw<false, 4> { using T = float4; };
+template <> struct WRaw<false, 1> { using T = float; };
+
+template <bool BF16, int VEC>
+__device__ __forceinline__ typename WRaw<BF16, VEC>::T load_w(const void *W, int64_t idx)
+{
+    using T = typename WRaw<BF16, VEC>::T;
+    if constexpr (BF16)
+        return *reinterpret_cast<const T *>(static_cast<const unsigned short *>(W) + idx);
+    else
+        return *reinterpret_cast<const T *>(static_cast<const float *>(W) + idx);
+}
+
+__device__ __forceinline__ void unpack_w(const uint2 &u, float (&w)[4])
+{
+    w[0] = bf16_lo(u.x); w[1] = bf16_hi(u.x); w[2] = bf16_lo(u.y); w[3] = bf16_hi(u.y);
+}
+__device__ __forceinline__ void unpack_w(const unsigned short &u, float (&w)[1])
+{
+    w[0] = __uint_as_float((unsigned)u << 16);
+}
+__device__ __forceinline__ void unpack_w(const float4 &f, float (&w)[4])
+{
+    w[0] = f.x; w[1] = f.y; w[2] = f.z; w[3] = f.w;
+}
+__device__ __forceinline__ void unpack_w(const float &f, float (&w)[1]) { w[0] = f; }
+
+template <bool BF16, int VEC>
+__device__ __forceinline__ void store_w(void *W, int64_t idx, const float (&w)[VEC])
+{
+    if constexpr (BF16 && VEC == 4) {
+        uint2 u;
+        u.x = (unsigned)f2bf(w[0]) | ((unsigned)f2bf(w[1]) << 16);
+        u.y = (unsigned)f2bf(w[2]) | ((unsigned)f2bf(w[3]) << 16);
+        *reinterpret_cast<uint2 *>(static_cast<unsigned short *>(W) + idx) = u;
+    } else if constexpr (BF16) {
+        static_cast<unsigned short *>(W)[idx] = f2bf(w[0]);
+    } else if constexpr (VEC == 4) {
+        *reinterpret_cast<float4 *>(static_cast<float *>(W) + idx) = make_float4(w[0], w[1], w[2], w[3]);
+    } else {
+        static_cast<float *>(W)[idx] = w[0];
+    }
+}
+
+// Pass 3: the update.  Same row ranges and column mapping as pass 1; each
+// CTA walks its rows from the last iteration block to the first.  The
+// column scales live in shared memory (D floats).
+template <int VEC, int CPT, int R, bool BF16>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__restrict__ r,
+              const float *__restrict__ c, const DevScalars *__restrict__ sc,
+              int64_t V, int D, int tpr, float inv_bc, float eps, float lr_signed, int variant)
+{
+    using F = typename Vec<VEC>::F;
+    using WT = typename WRaw<BF16, VEC>::T;
+    extern __shared__ float cs[];  // D column scales
+    const int DV = D / VEC;
+    const int tid = threadIdx.x;
+    const int rg = kThreads / tpr;
+    const int g = tid / tpr;
+    const int l = tid - g * tpr;
+    const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
+    const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+    const int64_t step = (int64_t)rg * R;
+    const int64_t nblocks = (row1 - row0 + step - 1) / step;
+
+    // column scale sqrt(chat_j / s) (FULL), sqrt(chat_j) (COL) or 1 (ROW)
+    const float inv_s = (variant == EMBER_VARIANT_FULL) ? sc->inv_s : 1.f;
+    for (int j = tid; j < D; j += kThreads)
+        cs[j] = (variant == EMBER_VARIANT_ROW) ? 1.f : sqrtf(c[j] * inv_bc * inv_s);
+    __syncthreads();
+
+    for (int64_t b = nblocks - 1; b >= 0; --b) {
+        const int64_t base = row0 + b * step;
+        F gv[R][CPT];
+        WT wr[R][CPT];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+#pragma unroll
+            for (int cc = 0; cc < CPT; ++cc) {
+                const int col = l + cc * tpr;
+                if (i < row1 && col < DV) {
+                    gv[k][cc] = load_g<VEC>(G + i * D + (int64_t)col * VEC);
+                    wr[k][cc] = load_w<BF16, VEC>(W, i * D + (int64_t)col * VEC);
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+            if (i >= row1)
+                continue;
+            const float rs = (variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(__ldg(r + i) * inv_bc);
+#pragma unroll
+            for (int cc = 0; cc < CPT; ++cc) {
+                const int col = l + cc * tpr;
+                if (col >= DV)
+                    continue;
+                float w[VEC];
+                unpack_w(wr[k][cc], w);
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const float den = fmaf(rs, cs[col * VEC + e], eps);
+                    const float u = comp(gv[k][cc], e) / den;
+                    w[e] = fmaf(lr_signed, u, w[e]);
+                }
+                store_w<BF16, VEC>(W, i * D + (int64_t)col * VEC, w);
+            }
+        }
+    }
+}
+
+template <int VEC, int CPT>
+cudaError_t launch_dense_t(const DenseArgs &a)
+{
+    constexpr int R1 = (16 / CPT) < 1 ? 1 : (16 / CPT);
+    constexpr int R3 = (4 / CPT) < 1 ? 1 : (4 / CPT);
+    const int nparts = (int)(a.V < kGridCtas ? a.V : kGridCtas);
+    const int D = (int)a.D;
+    DevScalars *sc = reinterpret_cast<DevScalars *>(a.ws + a.lay.scalars);
+    double *rsum_part = reinterpret_cast<double *>(a.ws + a.lay.rsum_part);
+    double *csum_part = reinterpret_cast<double *>(a.ws + a.lay.csum_part);
+    float *colpart = reinterpret_cast<float *>(a.ws + a.lay.colpart);
+    const int rg = kThreads / a.map.tpr;
+    const size_t shmem = (rg > 1) ? (size_t)D * sizeof(float) : 0;
+
+    if (a.trace)
+        cudaEventRecord(a.trace[0], a.stream);
+    k_reduce_dense<VEC, CPT, R1><<<nparts, kThreads, shmem, a.stream>>>(
+        a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2);
+    const int nstate = (D + kStateCols - 1) / kStateCols;
+    if (a.trace)
+        cudaEventRecord(a.trace[1], a.stream);
+    k_state_dense<<<nstate, kStateThreads, 0, a.stream>>>(
+        colpart, nparts, rsum_part, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2, a.inv_bc);
+    if (a.trace)
+        cudaEventRecord(a.trace[2], a.stream);
+    const size_t cs_bytes = (size_t)D * sizeof(float);
+    if (a.wbf16)
+        k_apply_dense<VEC, CPT, R3, true><<<nparts, kThreads, cs_bytes, a.stream>>>(
+            a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+    else
+        k_apply_dense<VEC, CPT, R3, false><<<nparts, kThreads, cs_bytes, a.stream>>>(
+            a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+    if (a.trace)
+        cudaEventRecord(a.trace[3], a.stream);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)
+{
+    const int vec = (vec4_ok && D % 4 == 0) ? 4 : 1;
+    const int64_t DV = D / vec;
+    for (int tpr = 32; tpr <= kThreads; tpr *= 2) {
+        const int64_t need = (DV + tpr - 1) / tpr;
+        if (need <= 4 || tpr == kThreads) {
+            int cpt = 1;
+            while (cpt < need)
+                cpt *= 2;
+            if (cpt > 8)
+                return false;
+            m->vec = vec;
+            m->tpr = tpr;
+            m->cpt = cpt;
+            return true;
+        }
+    }
+    return false;
+}
+
+cudaError_t launch_dense_step(const DenseArgs &a)
+{
+    if (a.map.vec == 4) {
+        switch (a.map.cpt) {
+        case 1: return launch_dense_t<4, 1>(a);
+        case 2: return launch_dense_t<4, 2>(a);
+        case 4: return launch_dense_t<4, 4>(a);
+        case 8: return launch_dense_t<4, 8>(a);
+        }
+    } else {
+        switch (a.map.cpt) {
+        case 1: return launch_dense_t<1, 1>(a);
+        case 2: return launch_dense_t<1, 2>(a);
+        case 4: return launch_dense_t<1, 4>(a);
+        case 8: return launch_dense_t<1, 8>(a);
+        }
+    }
+    return cudaErrorInvalidValue;
+}
+
+}  // namespace ember

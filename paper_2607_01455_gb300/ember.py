@@ -1,0 +1,234 @@
+"""ctypes binding of libember (include/ember.h), with the C names.
+
+Argument marshalling only: every step runs in the CUDA kernels of the
+library.  Pointers may be passed as integers or as torch tensors (their
+data_ptr() is used); streams as integers, torch.cuda.Stream objects or None
+(the current torch stream).  A non-OK status raises EmberError.  If the
+compiled library is missing this module raises on import of the library
+instead of falling back to anything else.
+"""
+import ctypes
+import os
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_HERE, "_lib", "libember.so")
+
+EMBER_OK = 0
+EMBER_ERR_INVALID_ARG = 1
+EMBER_ERR_ALIGNMENT = 2
+EMBER_ERR_DTYPE = 3
+EMBER_ERR_WORKSPACE = 4
+EMBER_ERR_CUDA = 5
+EMBER_ERR_ID_OUT_OF_RANGE = 6
+EMBER_ERR_TIMEOUT = 7
+EMBER_ERR_UNSUPPORTED = 8
+
+EMBER_F32 = 0
+EMBER_BF16 = 1
+EMBER_I32 = 0
+EMBER_I64 = 1
+EMBER_VARIANT_FULL = 0
+EMBER_VARIANT_ROW = 1
+EMBER_VARIANT_COL = 2
+
+# Every function include/ember.h declares.
+EXPORTS = (
+    "ember_hparams_default", "ember_create", "ember_destroy", "ember_state_numel",
+    "ember_workspace_bytes", "ember_bind_workspace", "ember_step_dense",
+    "ember_step_sparse", "ember_get_device_status", "ember_status_string",
+    "ember_abi_version", "ember_set_trace_events",
+)
+
+
+class ember_hparams(ctypes.Structure):
+    _fields_ = [("beta2", ctypes.c_double), ("eps", ctypes.c_double),
+                ("maximize", ctypes.c_int), ("bias_correction", ctypes.c_int),
+                ("variant", ctypes.c_int)]
+
+
+class EmberError(RuntimeError):
+    def __init__(self, status, where=""):
+        self.status = status
+        super().__init__(f"{where}: {ember_status_string(status)} (status {status})")
+
+
+_lib = None
+
+
+def lib():
+    """The loaded libember.so; raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                f"{LIB_PATH} is missing: build it with __graft_entry__.build() "
+                "(there is no fallback implementation)")
+        L = ctypes.CDLL(LIB_PATH)
+        vp, i64, sz, st, flt, ip = (ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t,
+                                    ctypes.c_int, ctypes.c_float, ctypes.c_int)
+        hp = ctypes.POINTER(ember_hparams)
+        sig = {
+            "ember_hparams_default": (None, [hp]),
+            "ember_create": (st, [i64, i64, hp, ip, ctypes.POINTER(vp)]),
+            "ember_destroy": (None, [vp]),
+            "ember_state_numel": (sz, [vp]),
+            "ember_workspace_bytes": (sz, [vp, i64]),
+            "ember_bind_workspace": (st, [vp, vp, sz, i64, vp]),
+            "ember_step_dense": (st, [vp, vp, vp, vp, flt, i64, vp]),
+            "ember_step_sparse": (st, [vp, vp, vp, ip, i64, vp, vp, flt, i64, vp]),
+            "ember_get_device_status": (st, [vp, vp]),
+            "ember_status_string": (ctypes.c_char_p, [st]),
+            "ember_abi_version": (ip, []),
+            "ember_set_trace_events": (st, [vp, ctypes.POINTER(vp), ip]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(L, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _addr(x):
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(s):
+    if s is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def _check(status, where):
+    if status != EMBER_OK:
+        raise EmberError(status, where)
+
+
+def ember_status_string(status):
+    return lib().ember_status_string(status).decode()
+
+
+def ember_abi_version():
+    return lib().ember_abi_version()
+
+
+def ember_hparams_default():
+    hp = ember_hparams()
+    lib().ember_hparams_default(ctypes.byref(hp))
+    return hp
+
+
+def ember_create(V, D, hparams=None, wdtype=EMBER_BF16):
+    """Returns the handle (an integer); raises EmberError on a bad argument."""
+    out = ctypes.c_void_p()
+    hp = ctypes.byref(hparams) if hparams is not None else None
+    _check(lib().ember_create(V, D, hp, wdtype, ctypes.byref(out)), "ember_create")
+    return out.value
+
+
+def ember_destroy(h):
+    lib().ember_destroy(h)
+
+
+def ember_state_numel(h):
+    return lib().ember_state_numel(h)
+
+
+def ember_workspace_bytes(h, max_sparse_N=0):
+    return lib().ember_workspace_bytes(h, max_sparse_N)
+
+
+def ember_bind_workspace(h, workspace, nbytes, max_sparse_N=0, stream=None):
+    _check(lib().ember_bind_workspace(h, _addr(workspace), nbytes, max_sparse_N, _stream(stream)),
+           "ember_bind_workspace")
+
+
+def ember_step_dense(h, W, G, state, lr, t, stream=None):
+    _check(lib().ember_step_dense(h, _addr(W), _addr(G), _addr(state), lr, t, _stream(stream)),
+           "ember_step_dense")
+
+
+def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
+    _check(lib().ember_step_sparse(h, _addr(W), _addr(ids), idtype, N, _addr(rows), _addr(state),
+                                   lr, t, _stream(stream)), "ember_step_sparse")
+
+
+def ember_get_device_status(h, stream=None):
+    """Synchronises the stream; returns (and clears) the sticky device status."""
+    return lib().ember_get_device_status(h, _stream(stream))
+
+
+def ember_set_trace_events(h, events):
+    """events: torch.cuda.Event objects (created with enable_timing=True) or raw
+    handles; [] stops tracing.  torch creates an event lazily, so each one is
+    recorded once here to make sure it exists."""
+    handles = []
+    for ev in events:
+        if isinstance(ev, int):
+            handles.append(ev)
+        else:
+            ev.record()
+            handles.append(ev.cuda_event)
+    arr = (ctypes.c_void_p * max(len(handles), 1))(*handles)
+    _check(lib().ember_set_trace_events(h, arr if handles else None, len(handles)),
+           "ember_set_trace_events")
+
+
+class Ember:
+    """One token table's optimizer: the handle, its fp32 state (r then c) and
+    its workspace, all device memory allocated through torch."""
+
+    def __init__(self, V, D, wdtype="bf16", beta2=0.999, eps=1e-8, maximize=False,
+                 bias_correction=True, variant="full", max_sparse_N=0, device="cuda"):
+        import torch
+        hp = ember_hparams(beta2=beta2, eps=eps, maximize=int(maximize),
+                           bias_correction=int(bias_correction),
+                           variant={"full": 0, "row": 1, "col": 2}[variant])
+        self.V, self.D = V, D
+        self.wdtype = {"bf16": EMBER_BF16, "f32": EMBER_F32}[wdtype]
+        self.handle = ember_create(V, D, hp, self.wdtype)
+        self.state = torch.zeros(ember_state_numel(self.handle), dtype=torch.float32, device=device)
+        nbytes = ember_workspace_bytes(self.handle, max_sparse_N)
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        self.max_sparse_N = max_sparse_N
+        ember_bind_workspace(self.handle, self.workspace, nbytes, max_sparse_N)
+
+    @property
+    def r(self):
+        return self.state[: self.V]
+
+    @property
+    def c(self):
+        return self.state[self.V:]
+
+    def step_dense(self, W, G, lr, t, stream=None):
+        ember_step_dense(self.handle, W, G, self.state, lr, t, stream)
+
+    def step_sparse(self, W, ids, rows, lr, t, stream=None):
+        import torch
+        idtype = EMBER_I64 if ids.dtype == torch.int64 else EMBER_I32
+        ember_step_sparse(self.handle, W, ids, idtype, ids.numel(), rows, self.state, lr, t, stream)
+
+    def trace(self, events):
+        ember_set_trace_events(self.handle, events)
+
+    def device_status(self, stream=None):
+        return ember_get_device_status(self.handle, stream)
+
+    def close(self):
+        if self.handle:
+            ember_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
