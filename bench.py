@@ -55,6 +55,58 @@ def kernel_bytes(wl):
     return {"reduce": 4 * V * D + 8 * V, "state": 8 * D, "apply": (4 + 2 * w) * V * D + 4 * (V + D)}
 
 
+def sparse_bytes(wl, U):
+    """Algorithmic bytes of one sparse step with U distinct ids: the grad
+    rows read once, the ids read once, the summed rows visited a second time
+    (written and read back, or the rows re-read, whichever is less), the
+    touched W rows read and written, r read and written for all V rows."""
+    N, D, V, w = wl.N, wl.D, wl.V, wbytes(wl)
+    return 4 * N * D + 8 * N + min(8 * U * D, 4 * N * D) + 2 * w * U * D + 8 * V + 8 * D
+
+
+SPARSE_KERNELS = ("tile_sort", "rank", "scatter", "heads", "segments", "chunks", "carry", "vpass",
+                  "state", "apply")
+
+
+def run_sparse(wl, dev, steps, warmup, flush, seed=0):
+    """Times the sparse step on one fixed batch (L2 flushed between steps)."""
+    import torch
+    from paper_2607_01455_gb300 import synth
+    from paper_2607_01455_gb300.ember import Ember
+    W = synth.init_weights(wl, seed, dev)
+    ids, rows = synth.sparse_batch(wl, seed, 1, dev)
+    U = int(torch.unique(ids).numel())
+    emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, max_sparse_N=wl.N, device=dev)
+    nk = len(SPARSE_KERNELS)
+    t = 0
+    warm = [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)]
+    for _ in range(warmup):
+        t += 1
+        flush.zero_()
+        emb.trace(warm)
+        emb.step_sparse(W, ids, rows, wl.lr, t)
+    torch.cuda.synchronize()
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(steps)]
+    for k in range(steps):
+        t += 1
+        flush.zero_()
+        emb.trace(events[k])
+        emb.step_sparse(W, ids, rows, wl.lr, t)
+    torch.cuda.synchronize()
+    emb.trace([])
+    if emb.device_status() != 0:
+        raise SystemExit("device status after the sparse steps")
+    per = {name: sum(ev[i].elapsed_time(ev[i + 1]) for ev in events) / steps
+           for i, name in enumerate(SPARSE_KERNELS)}
+    ms = sum(ev[0].elapsed_time(ev[nk]) for ev in events) / steps
+    B = sparse_bytes(wl, U)
+    return {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "unique_ids": U,
+            "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
+            "algorithmic_bytes": B, "touched_params_per_s": U * wl.D / (ms * 1e-3),
+            "occurrence_params_per_s": wl.N * wl.D / (ms * 1e-3),
+            "kernels_ms": per, "gpu_launches": nk * steps}
+
+
 def measured_hbm_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -64,7 +116,7 @@ def measured_hbm_peak():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -80,7 +132,7 @@ class ClockSampler:
             self.out = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "200"],
+                 "--format=csv,noheader,nounits", "-lms", "100"],
                 stdout=self.out, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -192,17 +244,54 @@ def run_reference(args, world, rank):
     return 0
 
 
+def sparse_kernel_bytes(wl, U):
+    """Algorithmic bytes per launch of the segment-sum kernel (grad rows read,
+    summed rows written, sorted order read) and of the apply kernel."""
+    N, D, w = wl.N, wl.D, wbytes(wl)
+    return {"chunks": 4 * N * D + 4 * U * D + 8 * N, "apply": 4 * U * D + 2 * w * U * D + 8 * U}
+
+
+def run_sparse_line(args, wl, world, rank, dev):
+    import torch
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    barrier(world)
+    with ClockSampler(dev.index or 0) as clocks:
+        sp = run_sparse(wl, dev, args.steps, args.warmup, flush, seed=rank)
+        barrier(world)
+    ms = allreduce_max(world, sp["ms_per_step"])
+    peak, peak_kind = measured_hbm_peak()
+    kb = sparse_kernel_bytes(wl, sp["unique_ids"])
+    ach = kb["chunks"] / (sp["kernels_ms"]["chunks"] * 1e-3) / 1e9
+    line = {
+        "metric": METRIC, "value": world * sp["algorithmic_bytes"] / (ms * 1e-3) / 1e9, "unit": "GB/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "w_dtype": wl.wdtype,
+                   "ids": "int64", "l2": "flushed between steps (512 MiB write, outside the events)",
+                   "parallelism": f"replicas x{world}"},
+        "roofline": {"bound": "hbm", "kernel": "k_sp_chunks", "achieved": ach, "peak": peak,
+                     "unit": "GB/s", "frac": ach / peak, "peak_kind": peak_kind, "traffic": None,
+                     "algorithmic_bytes_per_launch": kb["chunks"]},
+        "cpu_baseline": None, "e2e": None, "gpu_launches": sp["gpu_launches"],
+        "clocks": clocks.summary(), "sparse": sp,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
 def run_ours(args, world, rank, local):
     import torch
     from paper_2607_01455_gb300 import synth
     from paper_2607_01455_gb300.ember import Ember
 
     wl = synth.WORKLOADS[args.workload]
-    if wl.kind != "dense":
-        raise SystemExit("bench.py times the dense workloads")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
+    if wl.kind == "sparse":
+        return run_sparse_line(args, wl, world, rank, dev)
 
     W = synth.init_weights(wl, rank, dev)
     G = synth.dense_grad(wl, rank, 1, dev)
@@ -294,6 +383,13 @@ def run_ours(args, world, rank, local):
                "sample": f"3 oracle dense steps on the first {rows} of {wl.V} rows (D={wl.D}), one thread",
                "ms_per_step": sec * 1e3}
 
+    sparse = None
+    if not args.no_sparse:
+        swl = synth.WORKLOADS["sparse_v262144_d2048_bf16_n32768"]
+        sparse = run_sparse(swl, dev, max(10, min(args.steps, 100)), args.warmup, flush, seed=rank)
+        sparse["frac_of_nominal_8TBs"] = sparse["value"] / NOMINAL_HBM_GBS
+        sparse["frac_of_measured_hbm"] = sparse["value"] / peak
+
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -311,6 +407,7 @@ def run_ours(args, world, rank, local):
         "frac_of_measured_hbm": value / world / peak,
         "kernels": kern,
         "wall_s_timed_region": wall,
+        "sparse": sparse,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -320,12 +417,13 @@ def run_ours(args, world, rank, local):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--steps", type=int, default=400)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-sparse", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

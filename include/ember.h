@@ -146,6 +146,17 @@ ember_status ember_step_sparse(ember_handle *h, void *W, const void *ids,
                                ember_idtype idtype, int64_t N, const float *rows,
                                float *state, float lr, int64_t t, void *stream);
 
+/* Token-id dedup alone (the first part of ember_step_sparse, Section 2.2):
+ * writes, on `stream`, the distinct ids of ids[0..N) that lie in [0, V) in
+ * ascending order to uniq[0..U), how often each occurs to counts[0..U), and
+ * U to *n_unique.  uniq and counts hold N int32 each, n_unique one int32;
+ * all three are device memory owned by the caller.  Uses the bound
+ * workspace (N <= max_sparse_N); leaves the optimizer state untouched.
+ * Ids outside [0, V) are skipped and set EMBER_ERR_ID_OUT_OF_RANGE in the
+ * device flag. */
+ember_status ember_sparse_unique(ember_handle *h, const void *ids, ember_idtype idtype, int64_t N,
+                                 int32_t *uniq, int32_t *counts, int32_t *n_unique, void *stream);
+
 /* Synchronise `stream`, return the sticky device flag of this handle's
  * workspace (EMBER_OK if no device error happened since the last call) and
  * clear it. */

@@ -15,7 +15,6 @@ static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
 {
-    (void)V;
     Layout L{};
     size_t off = 0;
     auto take = [&](size_t bytes) {
@@ -27,15 +26,23 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
     L.scalars = take(sizeof(DevScalars));
     L.rsum_part = take(sizeof(double) * kGridCtas);
     L.csum_part = take(sizeof(double) * nstate);
-    L.colpart = take(sizeof(float) * (size_t)kGridCtas * (size_t)D);
+    L.colpart = take(sizeof(float) * 2 * (size_t)kGridCtas * (size_t)D);
     if (max_sparse_N > 0) {
         const size_t N = (size_t)max_sparse_N;
-        L.sp_keys = take(sizeof(uint64_t) * N);
+        const size_t Npad = (N + kSortTile - 1) / kSortTile * kSortTile;
+        const size_t nslices = (size_t)((D + kThreads - 1) / kThreads);
+        const size_t nchunks = (N + kChunk - 1) / kChunk;
+        L.sp_keys = take(sizeof(uint64_t) * Npad);
+        L.sp_rank = take(sizeof(int32_t) * Npad);
         L.sp_sorted = take(sizeof(uint64_t) * N);
-        L.sp_head = take(sizeof(int32_t) * (N + 1));
+        L.sp_tilecnt = take(sizeof(int32_t) * 2 * (Npad / kSortTile));
+        L.sp_perm = take(sizeof(int32_t) * N);
+        L.sp_segidx = take(sizeof(int32_t) * N);
         L.sp_uniq = take(sizeof(int32_t) * N);
         L.sp_segoff = take(sizeof(int32_t) * (N + 1));
-        L.sp_tilecnt = take(sizeof(int32_t) * (N + 2));
+        L.sp_slot = take(sizeof(int32_t) * (size_t)V);
+        L.sp_rowpart = take(sizeof(float) * N * nslices);
+        L.sp_carry = take(sizeof(float) * 2 * nchunks * (size_t)D);
         L.sp_rows = take(sizeof(float) * N * (size_t)D);
     }
     L.total = off;
@@ -135,6 +142,11 @@ ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes
     if (cudaMemsetAsync((unsigned char *)workspace + L.scalars, 0, sizeof(DevScalars),
                         (cudaStream_t)stream) != cudaSuccess)
         return EMBER_ERR_CUDA;
+    // the sparse step expects an all-zero slot map and leaves it all-zero
+    if (max_sparse_N > 0 &&
+        cudaMemsetAsync((unsigned char *)workspace + L.sp_slot, 0, sizeof(int32_t) * (size_t)h->V,
+                        (cudaStream_t)stream) != cudaSuccess)
+        return EMBER_ERR_CUDA;
     h->ws = (unsigned char *)workspace;
     h->ws_bytes = bytes;
     h->ws_max_N = max_sparse_N;
@@ -182,14 +194,75 @@ ember_status ember_step_sparse(ember_handle *h, void *W, const void *ids, ember_
                                int64_t N, const float *rows, float *state, float lr, int64_t t,
                                void *stream)
 {
-    (void)stream;
     if (!h || !W || !state || N < 0 || (N > 0 && (!ids || !rows)))
         return EMBER_ERR_INVALID_ARG;
     if (t < 1 || !isfinite(lr))
         return EMBER_ERR_INVALID_ARG;
     if (idtype != EMBER_I32 && idtype != EMBER_I64)
         return EMBER_ERR_DTYPE;
-    return EMBER_ERR_UNSUPPORTED;
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    const size_t isz = idtype == EMBER_I64 ? 8 : 4;
+    if (!is_aligned(W, wsz) || !is_aligned(state, 4) || (N > 0 && (!is_aligned(ids, isz) ||
+                                                                  !is_aligned(rows, 4))))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    if (N > h->ws_max_N)
+        return EMBER_ERR_WORKSPACE;
+
+    SparseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.N = N;
+    a.wbf16 = h->wdtype == EMBER_BF16;
+    a.ids64 = idtype == EMBER_I64;
+    a.W = W;
+    a.ids = ids;
+    a.rows = rows;
+    a.r = state;
+    a.c = state + h->V;
+    a.beta2 = h->hp.beta2;
+    a.one_minus_beta2 = 1.0 - h->hp.beta2;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.eps = (float)h->hp.eps;
+    a.variant = h->hp.variant;
+    a.ws = h->ws;
+    a.lay = make_layout(h->V, h->D, h->ws_max_N);
+    a.stream = (cudaStream_t)stream;
+    a.trace = h->n_trace > 0 ? h->trace : nullptr;
+    a.n_trace = h->n_trace;
+    const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && (N == 0 || is_aligned(rows, 16));
+    if (!choose_colmap(h->D, vec4, &a.map))
+        return EMBER_ERR_UNSUPPORTED;
+    return launch_sparse_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+ember_status ember_sparse_unique(ember_handle *h, const void *ids, ember_idtype idtype, int64_t N,
+                                 int32_t *uniq, int32_t *counts, int32_t *n_unique, void *stream)
+{
+    if (!h || N < 0 || (N > 0 && (!ids || !uniq || !counts)) || !n_unique)
+        return EMBER_ERR_INVALID_ARG;
+    if (idtype != EMBER_I32 && idtype != EMBER_I64)
+        return EMBER_ERR_DTYPE;
+    const size_t isz = idtype == EMBER_I64 ? 8 : 4;
+    if ((N > 0 && (!is_aligned(ids, isz) || !is_aligned(uniq, 4) || !is_aligned(counts, 4))) ||
+        !is_aligned(n_unique, 4))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    if (N > h->ws_max_N)
+        return EMBER_ERR_WORKSPACE;
+    SparseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.N = N;
+    a.ids64 = idtype == EMBER_I64;
+    a.ids = ids;
+    a.ws = h->ws;
+    a.lay = make_layout(h->V, h->D, h->ws_max_N);
+    a.stream = (cudaStream_t)stream;
+    return launch_sparse_unique(a, uniq, counts, n_unique) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
 }
 
 ember_status ember_get_device_status(ember_handle *h, void *stream)

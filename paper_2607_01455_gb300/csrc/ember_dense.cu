@@ -31,75 +31,13 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "ember_device.cuh"
 #include "ember_internal.h"
 
 namespace ember {
 namespace {
 
-template <int VEC> struct Vec;
-template <> struct Vec<4> { using F = float4; };
-template <> struct Vec<1> { using F = float; };
-
-__device__ __forceinline__ float comp(const float4 &v, int e)
-{
-    return e == 0 ? v.x : e == 1 ? v.y : e == 2 ? v.z : v.w;
-}
-__device__ __forceinline__ float comp(const float &v, int) { return v; }
-__device__ __forceinline__ void set_comp(float4 &v, int e, float x)
-{
-    if (e == 0) v.x = x; else if (e == 1) v.y = x; else if (e == 2) v.z = x; else v.w = x;
-}
-__device__ __forceinline__ void set_comp(float &v, int, float x) { v = x; }
-
-template <int VEC>
-__device__ __forceinline__ typename Vec<VEC>::F load_g(const float *p)
-{
-    if constexpr (VEC == 4)
-        return __ldg(reinterpret_cast<const float4 *>(p));
-    else
-        return __ldg(p);
-}
-
-template <int VEC>
-__device__ __forceinline__ typename Vec<VEC>::F zero_vec()
-{
-    if constexpr (VEC == 4)
-        return make_float4(0.f, 0.f, 0.f, 0.f);
-    else
-        return 0.f;
-}
-
-// Sum R per-lane values over the 32 lanes of a warp, "transposed": each
-// halving step trades half of the values with a partner lane, so the R
-// totals cost R-1 + log2(32/R) shuffles instead of 5R.  On return v[0] of
-// lane l is the warp total of value index `row` (lanes whose low
-// log2(32/R) bits differ hold the same total).  The addition tree is fixed,
-// so the result is the same on every run.
-template <int R>
-__device__ __forceinline__ float warp_sum_transposed(float (&v)[R], int lane, int &row)
-{
-    static_assert(R >= 1 && R <= 32 && (R & (R - 1)) == 0, "R must be a power of two <= 32");
-    constexpr int kLog = (R >= 32) ? 5 : (R >= 16) ? 4 : (R >= 8) ? 3 : (R >= 4) ? 2 : (R >= 2) ? 1 : 0;
-    row = 0;
-#pragma unroll
-    for (int s = 0; s < kLog; ++s) {
-        const int o = 16 >> s;
-        const int h = R >> (s + 1);
-        const bool hi = (lane & o) != 0;
-#pragma unroll
-        for (int m = 0; m < h; ++m) {
-            const float send = hi ? v[m] : v[m + h];
-            const float keep = hi ? v[m + h] : v[m];
-            v[m] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-        if (hi)
-            row += h;
-    }
-#pragma unroll
-    for (int o = 16 >> kLog; o >= 1; o >>= 1)
-        v[0] += __shfl_xor_sync(0xffffffffu, v[0], o);
-    return v[0];
-}
+using namespace dev;
 
 // Pass 1: one read of G.  Template: VEC columns per access, CPT accesses per
 // thread per row, R rows per row group per iteration.
@@ -245,7 +183,7 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
 // [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in order.
 __global__ void __launch_bounds__(kStateThreads)
 k_state_dense(const float *__restrict__ colpart, int nparts, const double *__restrict__ rsum_part,
-              float *__restrict__ c, double *__restrict__ csum_part, DevScalars *sc,
+              int nrsum, float *__restrict__ c, double *__restrict__ csum_part, DevScalars *sc,
               int64_t V, int D, double beta2, double one_minus_beta2, double inv_bc)
 {
     constexpr int kW = kStateThreads / 32;
@@ -255,10 +193,21 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
     __shared__ double part[kW][32];
     __shared__ bool am_last;
 
+    // rows w, w + 8, w + 16, ... in that order; eight loads in flight at a time
+    constexpr int kBatch = 8;
     double acc = 0.0;
     if (j < D)
-        for (int b = w; b < nparts; b += kW)
-            acc += (double)colpart[(int64_t)b * D + j];
+        for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
+            float v[kBatch];
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k) {
+                const int b = b0 + k * kW;
+                v[k] = (b < nparts) ? __ldcg(colpart + (int64_t)b * D + j) : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < kBatch; ++k)
+                acc += (double)v[k];
+        }
     part[w][lane] = acc;
     __syncthreads();
     if (w == 0) {
@@ -279,21 +228,27 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
         if (lane == 0)
             csum_part[blockIdx.x] = cn;
     }
+    double csum = 0.0, rsum = 0.0;
     if (threadIdx.x == 0) {
         __threadfence();
         const unsigned t = atomicAdd(&sc->ticket, 1u);
         am_last = (t == gridDim.x - 1);
     }
     __syncthreads();
-    if (am_last && threadIdx.x == 0) {
+    if (am_last && w == 0) {
         __threadfence();
-        const volatile double *cp = csum_part;
-        double csum = 0.0;
-        for (int b = 0; b < (int)gridDim.x; ++b)
-            csum += cp[b];
-        double rsum = 0.0;
-        for (int b = 0; b < nparts; ++b)
-            rsum += rsum_part[b];
+        // lane l sums entries l, l + 32, ... in order, then a fixed butterfly
+        for (int b = lane; b < (int)gridDim.x; b += 32)
+            csum += __ldcg(csum_part + b);
+        for (int b = lane; b < nrsum; b += 32)
+            rsum += __ldcg(rsum_part + b);
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) {
+            csum += __shfl_xor_sync(0xffffffffu, csum, o);
+            rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+        }
+    }
+    if (am_last && threadIdx.x == 0) {
         const double rbar = rsum * inv_bc / (double)V;
         const double cbar = csum * inv_bc / (double)D;
         const double s = sqrt(rbar * cbar);
@@ -302,61 +257,6 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
         sc->cbar = cbar;
         sc->inv_s = (s > 0.0) ? (float)(1.0 / s) : 0.f;
         sc->ticket = 0u;
-    }
-}
-
-__device__ __forceinline__ float bf16_lo(unsigned u) { return __uint_as_float(u << 16); }
-__device__ __forceinline__ float bf16_hi(unsigned u) { return __uint_as_float(u & 0xFFFF0000u); }
-__device__ __forceinline__ unsigned short f2bf(float x)
-{
-    return __bfloat16_as_ushort(__float2bfloat16_rn(x));
-}
-
-// Raw weight vectors: kept packed between the load and the update.
-template <bool BF16, int VEC> struct WRaw;
-template <> struct WRaw<true, 4> { using T = uint2; };
-template <> struct WRaw<true, 1> { using T = unsigned short; };
-template <> struct WRaw<false, 4> { using T = float4; };
-template <> struct WRaw<false, 1> { using T = float; };
-
-template <bool BF16, int VEC>
-__device__ __forceinline__ typename WRaw<BF16, VEC>::T load_w(const void *W, int64_t idx)
-{
-    using T = typename WRaw<BF16, VEC>::T;
-    if constexpr (BF16)
-        return *reinterpret_cast<const T *>(static_cast<const unsigned short *>(W) + idx);
-    else
-        return *reinterpret_cast<const T *>(static_cast<const float *>(W) + idx);
-}
-
-__device__ __forceinline__ void unpack_w(const uint2 &u, float (&w)[4])
-{
-    w[0] = bf16_lo(u.x); w[1] = bf16_hi(u.x); w[2] = bf16_lo(u.y); w[3] = bf16_hi(u.y);
-}
-__device__ __forceinline__ void unpack_w(const unsigned short &u, float (&w)[1])
-{
-    w[0] = __uint_as_float((unsigned)u << 16);
-}
-__device__ __forceinline__ void unpack_w(const float4 &f, float (&w)[4])
-{
-    w[0] = f.x; w[1] = f.y; w[2] = f.z; w[3] = f.w;
-}
-__device__ __forceinline__ void unpack_w(const float &f, float (&w)[1]) { w[0] = f; }
-
-template <bool BF16, int VEC>
-__device__ __forceinline__ void store_w(void *W, int64_t idx, const float (&w)[VEC])
-{
-    if constexpr (BF16 && VEC == 4) {
-        uint2 u;
-        u.x = (unsigned)f2bf(w[0]) | ((unsigned)f2bf(w[1]) << 16);
-        u.y = (unsigned)f2bf(w[2]) | ((unsigned)f2bf(w[3]) << 16);
-        *reinterpret_cast<uint2 *>(static_cast<unsigned short *>(W) + idx) = u;
-    } else if constexpr (BF16) {
-        static_cast<unsigned short *>(W)[idx] = f2bf(w[0]);
-    } else if constexpr (VEC == 4) {
-        *reinterpret_cast<float4 *>(static_cast<float *>(W) + idx) = make_float4(w[0], w[1], w[2], w[3]);
-    } else {
-        static_cast<float *>(W)[idx] = w[0];
     }
 }
 
@@ -447,11 +347,10 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         cudaEventRecord(a.trace[0], a.stream);
     k_reduce_dense<VEC, CPT, R1><<<nparts, kThreads, shmem, a.stream>>>(
         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2);
-    const int nstate = (D + kStateCols - 1) / kStateCols;
     if (a.trace)
         cudaEventRecord(a.trace[1], a.stream);
-    k_state_dense<<<nstate, kStateThreads, 0, a.stream>>>(
-        colpart, nparts, rsum_part, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2, a.inv_bc);
+    launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                 a.one_minus_beta2, a.inv_bc, a.stream);
     if (a.trace)
         cudaEventRecord(a.trace[2], a.stream);
     const size_t cs_bytes = (size_t)D * sizeof(float);
@@ -467,6 +366,15 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 }
 
 }  // namespace
+
+void launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum, float *c,
+                  double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                  double one_minus_beta2, double inv_bc, cudaStream_t stream)
+{
+    const int nstate = (D + kStateCols - 1) / kStateCols;
+    k_state_dense<<<nstate, kStateThreads, 0, stream>>>(colpart, nparts, rsum_part, nrsum, c, csum_part,
+                                                        sc, V, D, beta2, one_minus_beta2, inv_bc);
+}
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)
 {

@@ -41,20 +41,32 @@ struct DevScalars {
     int32_t n_valid;   // sparse step: number of ids inside [0, V)
 };
 
+// Sparse step: ids are sorted in tiles of kSortTile keys by kSortThreads
+// threads; the sorted occurrences are summed in chunks of kChunk.
+constexpr int kSortTile = 4096;
+constexpr int kSortThreads = 1024;
+constexpr int kChunk = 64;
+
 // Workspace layout (byte offsets, each 256-byte aligned).
 struct Layout {
     size_t scalars;     // DevScalars
     size_t rsum_part;   // double[kGridCtas]            sum of new r per CTA
     size_t csum_part;   // double[ceil(D/32)]           sum of new c per state CTA
-    size_t colpart;     // float[kGridCtas * D]         column sums of g^2 per CTA
-    // sparse step (present when max_sparse_N > 0)
-    size_t sp_keys;     // uint64[N]  (id << 32 | occurrence), tile-sorted
-    size_t sp_sorted;   // uint64[N]  globally sorted keys
-    size_t sp_head;     // int32[N + 1] run-head flags / offsets scratch
-    size_t sp_uniq;     // int32[N]   distinct ids, ascending
-    size_t sp_segoff;   // int32[N + 1] start of each distinct id's run in sp_sorted
-    size_t sp_tilecnt;  // int32[ceil(N / tile) + 1] per-tile counts
-    size_t sp_rows;     // float[N * D] summed gradient rows, one per distinct id
+    size_t colpart;     // float[2 * kGridCtas * D]     column sums of g^2 per CTA
+    // sparse step (present when max_sparse_N > 0); N = max_sparse_N,
+    // Npad = N rounded up to kSortTile
+    size_t sp_keys;     // uint64[Npad]  (id << 32 | occurrence), sorted within tiles
+    size_t sp_rank;     // int32[Npad]   global rank of each tile-sorted key
+    size_t sp_sorted;   // uint64[N]     keys in (id, occurrence) order
+    size_t sp_tilecnt;  // int32[2 * Npad / kSortTile]  heads and valid ids per tile
+    size_t sp_perm;     // int32[N]      occurrence index at each sorted position
+    size_t sp_segidx;   // int32[N]      distinct-id index at each sorted position
+    size_t sp_uniq;     // int32[N]      distinct ids, ascending
+    size_t sp_segoff;   // int32[N + 1]  first sorted position of each distinct id
+    size_t sp_slot;     // int32[V]      1 + distinct-id index of a touched row, else 0
+    size_t sp_rowpart;  // float[N * ceil(D / kThreads)]  sum g^2 per (distinct id, slice)
+    size_t sp_carry;    // float[2 * ceil(N / kChunk) * D]  partial sums of cut segments
+    size_t sp_rows;     // float[N * D]  summed gradient row of each distinct id
     size_t total;
 };
 
@@ -89,6 +101,37 @@ struct DenseArgs {
 };
 
 cudaError_t launch_dense_step(const DenseArgs &a);
+
+void launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum, float *c,
+                  double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                  double one_minus_beta2, double inv_bc, cudaStream_t stream);
+
+struct SparseArgs {
+    int64_t V, D, N;
+    int wbf16;
+    int ids64;
+    void *W;
+    const void *ids;
+    const float *rows;
+    float *r;
+    float *c;
+    double beta2, one_minus_beta2, inv_bc;
+    float lr_signed;
+    float eps;
+    int variant;
+    unsigned char *ws;
+    Layout lay;
+    ColMap map;
+    cudaStream_t stream;
+    const cudaEvent_t *trace;  // nullptr, or events to record at kernel boundaries
+    int n_trace;
+};
+
+cudaError_t launch_sparse_step(const SparseArgs &a);
+
+// Sort and dedup only; then copy the distinct ids, their counts and U out.
+cudaError_t launch_sparse_unique(const SparseArgs &a, int32_t *uniq_out, int32_t *counts_out,
+                                 int32_t *n_unique_out);
 
 constexpr int kMaxTraceEvents = 16;
 

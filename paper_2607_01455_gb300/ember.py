@@ -36,7 +36,7 @@ EXPORTS = (
     "ember_hparams_default", "ember_create", "ember_destroy", "ember_state_numel",
     "ember_workspace_bytes", "ember_bind_workspace", "ember_step_dense",
     "ember_step_sparse", "ember_get_device_status", "ember_status_string",
-    "ember_abi_version", "ember_set_trace_events",
+    "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
 )
 
 
@@ -80,6 +80,7 @@ def lib():
             "ember_status_string": (ctypes.c_char_p, [st]),
             "ember_abi_version": (ip, []),
             "ember_set_trace_events": (st, [vp, ctypes.POINTER(vp), ip]),
+            "ember_sparse_unique": (st, [vp, vp, ip, i64, vp, vp, vp, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -160,6 +161,11 @@ def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
                                    lr, t, _stream(stream)), "ember_step_sparse")
 
 
+def ember_sparse_unique(h, ids, idtype, N, uniq, counts, n_unique, stream=None):
+    _check(lib().ember_sparse_unique(h, _addr(ids), idtype, N, _addr(uniq), _addr(counts),
+                                     _addr(n_unique), _stream(stream)), "ember_sparse_unique")
+
+
 def ember_get_device_status(h, stream=None):
     """Synchronises the stream; returns (and clears) the sticky device status."""
     return lib().ember_get_device_status(h, _stream(stream))
@@ -215,6 +221,18 @@ class Ember:
         import torch
         idtype = EMBER_I64 if ids.dtype == torch.int64 else EMBER_I32
         ember_step_sparse(self.handle, W, ids, idtype, ids.numel(), rows, self.state, lr, t, stream)
+
+    def unique(self, ids, stream=None):
+        """(uniq, counts) of the valid ids, as int32 device tensors."""
+        import torch
+        idtype = EMBER_I64 if ids.dtype == torch.int64 else EMBER_I32
+        n = ids.numel()
+        uniq = torch.empty(max(n, 1), dtype=torch.int32, device=self.state.device)
+        counts = torch.empty(max(n, 1), dtype=torch.int32, device=self.state.device)
+        nu = torch.empty(1, dtype=torch.int32, device=self.state.device)
+        ember_sparse_unique(self.handle, ids, idtype, n, uniq, counts, nu, stream)
+        U = int(nu.item())
+        return uniq[:U], counts[:U]
 
     def trace(self, events):
         ember_set_trace_events(self.handle, events)
