@@ -132,6 +132,26 @@ ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes
 ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *state,
                               float lr, int64_t t, void *stream);
 
+/* The dense step for callers that cannot give the library any device
+ * memory: hosts whose allocator offers plugins no allocation hook,
+ * optimizer loops under a fully reserved memory budget, and code paths
+ * where a cudaMalloc would synchronise the device mid-step.  The paper has
+ * no counterpart; this is an interface convenience.
+ *   Same arguments, same kernels and same results as ember_step_dense, but
+ * no workspace is bound or used: the scratch (column and row-sum partials,
+ * scalars) lives in a 10 MiB array inside the library, present on every GPU
+ * that loads the library until the process exits.  Nothing is allocated.
+ * Every table this library accepts fits (D <= 8192 needs 9.97 MB); a larger
+ * need returns EMBER_ERR_WORKSPACE.
+ *   The first call on each device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture.  All calls on a device share the one array and
+ * each starts by zeroing its scalars, so calls that overlap on the GPU (two
+ * streams, two handles, two threads) race and must be serialised by the
+ * caller. */
+ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const float *G, float *state,
+                                      float lr, int64_t t, void *stream);
+
 /* One sparse Ember step (Section 2.2) at step number t >= 1.
  *   ids:   N token ids of type idtype (duplicates allowed, any order).
  *   rows:  N x D fp32, row k is the gradient contribution of occurrence k

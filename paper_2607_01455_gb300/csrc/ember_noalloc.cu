@@ -1,0 +1,109 @@
+// ember_step_dense_noalloc: the dense step with library-owned scratch.
+//
+// Some callers cannot hand this library a device workspace:
+//   - hosts whose device memory is owned by a framework allocator that
+//     gives plugins no allocation hook;
+//   - optimizer loops running under a fixed memory budget that is already
+//     fully reserved;
+//   - code paths where a cudaMalloc would synchronise the device in the
+//     middle of a training step.
+// For them this entry point runs the very same three kernels as
+// ember_step_dense, with their scratch (per-CTA column partials, row-sum
+// partials, a few scalars) in a file-scope device array instead of a bound
+// workspace.  It allocates nothing: no cudaMalloc, no cudaFree, no allocating
+// library call.
+//
+// The array is kNoAllocScratchBytes (10 MiB) on every GPU that loads the
+// library, held until the process exits.  That covers every table width the
+// dense step supports (D <= 8192 needs 9.97 MB); a larger need is refused.
+//
+// In host code the array's name is only a host-side stand-in; the kernels get
+// its device address, looked up once per device with cudaGetSymbolAddress on
+// the first call made with that device current.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <mutex>
+#include <stdint.h>
+
+#include "ember_internal.h"
+
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = size_t(10) << 20;
+constexpr int kMaxDevices = 64;
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
+
+std::mutex g_setup_mutex;
+unsigned char *g_scratch_addr[kMaxDevices] = {};
+
+// Device address of the scratch array on the current device (nullptr on error).
+unsigned char *scratch_for_current_device()
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
+        return nullptr;
+    std::lock_guard<std::mutex> lock(g_setup_mutex);
+    if (!g_scratch_addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
+            return nullptr;
+        g_scratch_addr[dev] = static_cast<unsigned char *>(p);
+    }
+    return g_scratch_addr[dev];
+}
+
+bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+}  // namespace
+
+extern "C" ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const float *G,
+                                                 float *state, float lr, int64_t t, void *stream)
+{
+    using namespace ember;
+    if (!h || !W || !G || !state)
+        return EMBER_ERR_INVALID_ARG;
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    if (!aligned(W, wsz) || !aligned(G, 4) || !aligned(state, 4))
+        return EMBER_ERR_ALIGNMENT;
+
+    // The dense kernels use the workspace's scalars, row-sum partials,
+    // column-sum partials of one CTA grid, nothing after that.
+    const Layout lay = make_layout(h->V, h->D, 0);
+    const size_t need = lay.colpart + sizeof(float) * (size_t)kGridCtas * (size_t)h->D;
+    if (need > kNoAllocScratchBytes)
+        return EMBER_ERR_WORKSPACE;
+
+    unsigned char *scratch = scratch_for_current_device();
+    if (!scratch)
+        return EMBER_ERR_CUDA;
+    cudaStream_t s = (cudaStream_t)stream;
+    // every call shares the array: start each one from zeroed scalars
+    if (cudaMemsetAsync(scratch + lay.scalars, 0, sizeof(DevScalars), s) != cudaSuccess)
+        return EMBER_ERR_CUDA;
+
+    DenseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.wbf16 = h->wdtype == EMBER_BF16;
+    a.W = W;
+    a.G = G;
+    a.r = state;
+    a.c = state + h->V;
+    a.beta2 = h->hp.beta2;
+    a.one_minus_beta2 = 1.0 - h->hp.beta2;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.eps = (float)h->hp.eps;
+    a.variant = h->hp.variant;
+    a.ws = scratch;
+    a.lay = lay;
+    a.stream = s;
+    a.trace = nullptr;
+    const bool vec4 = (h->D % 4 == 0) && aligned(W, 4 * wsz) && aligned(G, 16);
+    if (!choose_colmap(h->D, vec4, &a.map))
+        return EMBER_ERR_UNSUPPORTED;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}

@@ -37,6 +37,7 @@ EXPORTS = (
     "ember_workspace_bytes", "ember_bind_workspace", "ember_step_dense",
     "ember_step_sparse", "ember_get_device_status", "ember_status_string",
     "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
+    "ember_step_dense_noalloc",
 )
 
 
@@ -81,6 +82,7 @@ def lib():
             "ember_abi_version": (ip, []),
             "ember_set_trace_events": (st, [vp, ctypes.POINTER(vp), ip]),
             "ember_sparse_unique": (st, [vp, vp, ip, i64, vp, vp, vp, vp]),
+            "ember_step_dense_noalloc": (st, [vp, vp, vp, vp, flt, i64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -154,6 +156,12 @@ def ember_bind_workspace(h, workspace, nbytes, max_sparse_N=0, stream=None):
 def ember_step_dense(h, W, G, state, lr, t, stream=None):
     _check(lib().ember_step_dense(h, _addr(W), _addr(G), _addr(state), lr, t, _stream(stream)),
            "ember_step_dense")
+
+
+def ember_step_dense_noalloc(h, W, G, state, lr, t, stream=None):
+    """The dense step with the library's own scratch array (no workspace)."""
+    _check(lib().ember_step_dense_noalloc(h, _addr(W), _addr(G), _addr(state), lr, t,
+                                          _stream(stream)), "ember_step_dense_noalloc")
 
 
 def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
