@@ -60,8 +60,10 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
     const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
 
-    __shared__ float red[2][kWarps][R];
-    __shared__ double rsum_sh[kThreads];
+    // per-warp row sums of up to kRowBuf rows, finalised together
+    constexpr int kRowBuf = 128;
+    __shared__ float red[kWarps][kRowBuf];
+    __shared__ double rsum_sh[kWarps];
 
     float acc[CPT][VEC];
 #pragma unroll
@@ -71,8 +73,11 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
             acc[c][e] = 0.f;
     double rsum = 0.0;
 
-    int buf = 0;
-    for (int64_t base = row0; base < row1; base += (int64_t)rg * R, buf ^= 1) {
+    const int rows_per_it = rg * R;               // rows of one iteration
+    const int its_per_buf = kRowBuf / rows_per_it;  // >= 1: rg * R <= 128
+    int64_t buf_base = row0;
+    int nbuf = 0;  // iterations held in the buffer
+    for (int64_t base = row0; base < row1; base += rows_per_it) {
         F v[R][CPT];
 #pragma unroll
         for (int k = 0; k < R; ++k) {
@@ -116,26 +121,32 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
             for (int e = 0; e < VEC; ++e)
                 acc[c][e] += comp(v[0][c], e);
 
-        // row sums: within the warp, then across the warps of the row group
+        // row sums within the warp; buffered until the cross-warp step
         int row_in_warp;
         const float tot = warp_sum_transposed<R>(rp, lane, row_in_warp);
         if ((lane & (32 / R - 1)) == 0)
-            red[buf][warp][row_in_warp] = tot;
-        __syncthreads();
-        if (l < R) {
-            const int64_t i = base + (int64_t)g * R + l;
-            if (i < row1) {
-                float sum = 0.f;
-                for (int q = 0; q < wpg; ++q)
-                    sum += red[buf][g * wpg + q][l];
-                const double mean_row = (double)sum / (double)D;
-                const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
-                r[i] = rn;
-                rsum += (double)rn;
+            red[warp][nbuf * rows_per_it + g * R + row_in_warp] = tot;
+        ++nbuf;
+        if (nbuf == its_per_buf || base + rows_per_it >= row1) {
+            __syncthreads();
+            // row buf_base + q: sum of its row group's warps, in warp order
+            for (int q = tid; q < nbuf * rows_per_it; q += kThreads) {
+                const int64_t i = buf_base + q;
+                if (i < row1) {
+                    const int gq = (q % rows_per_it) / R;
+                    float sum = 0.f;
+                    for (int k = 0; k < wpg; ++k)
+                        sum += red[gq * wpg + k][q];
+                    const double mean_row = (double)sum / (double)D;
+                    const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
+                    r[i] = rn;
+                    rsum += (double)rn;
+                }
             }
+            __syncthreads();
+            buf_base += (int64_t)nbuf * rows_per_it;
+            nbuf = 0;
         }
-        // the next iteration writes the other buffer; the one after that
-        // writes this buffer again only after the next __syncthreads().
     }
 
     // column partial of this CTA: row groups combined in order 0 .. rg-1
@@ -168,12 +179,16 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
             out[j] = colsh[j];
     }
 
-    // sum of the new r values of this CTA, threads in order
-    rsum_sh[tid] = rsum;
+    // sum of the new r values of this CTA: fixed butterfly per warp, warps in order
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+    if (lane == 0)
+        rsum_sh[warp] = rsum;
     __syncthreads();
     if (tid == 0) {
         double s = 0.0;
-        for (int q = 0; q < kThreads; ++q)
+        for (int q = 0; q < kWarps; ++q)
             s += rsum_sh[q];
         rsum_part[blockIdx.x] = s;
     }
@@ -193,8 +208,9 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
     __shared__ double part[kW][32];
     __shared__ bool am_last;
 
-    // rows w, w + 8, w + 16, ... in that order; eight loads in flight at a time
-    constexpr int kBatch = 8;
+    // rows w, w + 8, w + 16, ...: sixteen loads in flight, summed pairwise
+    // in fp32 within the batch and in fp64 across batches
+    constexpr int kBatch = 16;
     double acc = 0.0;
     if (j < D)
         for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
@@ -205,8 +221,11 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
                 v[k] = (b < nparts) ? __ldcg(colpart + (int64_t)b * D + j) : 0.f;
             }
 #pragma unroll
-            for (int k = 0; k < kBatch; ++k)
-                acc += (double)v[k];
+            for (int h = kBatch / 2; h >= 1; h >>= 1)
+#pragma unroll
+                for (int k = 0; k < h; ++k)
+                    v[k] += v[k + h];
+            acc += (double)v[0];
         }
     part[w][lane] = acc;
     __syncthreads();
@@ -333,7 +352,7 @@ template <int VEC, int CPT>
 cudaError_t launch_dense_t(const DenseArgs &a)
 {
     constexpr int R1 = (16 / CPT) < 1 ? 1 : (16 / CPT);
-    constexpr int R3 = (4 / CPT) < 1 ? 1 : (4 / CPT);
+    constexpr int R3 = (8 / CPT) < 1 ? 1 : (8 / CPT);
     const int nparts = (int)(a.V < kGridCtas ? a.V : kGridCtas);
     const int D = (int)a.D;
     DevScalars *sc = reinterpret_cast<DevScalars *>(a.ws + a.lay.scalars);

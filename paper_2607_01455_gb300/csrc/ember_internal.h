@@ -43,9 +43,9 @@ struct DevScalars {
 
 // Sparse step: ids are sorted in tiles of kSortTile keys by kSortThreads
 // threads; the sorted occurrences are summed in chunks of kChunk.
-constexpr int kSortTile = 4096;
-constexpr int kSortThreads = 1024;
-constexpr int kChunk = 64;
+constexpr int kSortTile = 1024;
+constexpr int kSortThreads = 256;
+constexpr int kChunk = 32;
 
 // Workspace layout (byte offsets, each 256-byte aligned).
 struct Layout {

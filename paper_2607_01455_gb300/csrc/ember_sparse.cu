@@ -14,7 +14,7 @@
 // Kernels, in launch order:
 //   sort      k_sp_tile_sort, k_sp_rank, k_sp_scatter: the N keys
 //             (id << 32 | occurrence) in ascending order, without atomics on
-//             floating-point data: 4096-key tiles are bitonic-sorted in shared
+//             floating-point data: 1024-key tiles are bitonic-sorted in shared
 //             memory, then every key's global rank is its rank in its tile
 //             plus its lower bound in every other tile (integer atomics, so
 //             the rank is exact and the order deterministic).
@@ -24,7 +24,7 @@
 //   segsum    k_sp_chunks, k_sp_carry: the summed gradient row of every
 //             distinct id, adding its occurrences in increasing occurrence
 //             order; per (id, column slice) sums of g^2; per-CTA column sums
-//             of g^2.  The sorted occurrences are cut into chunks of 64 so the
+//             of g^2.  The sorted occurrences are cut into chunks of 32 so the
 //             work is even however skewed the id counts are (a Zipf head id
 //             can own thousands of occurrences); a run that crosses chunk
 //             boundaries is summed piecewise and its pieces are added in
@@ -73,14 +73,15 @@ k_sp_tile_sort(const IdT *__restrict__ ids, int64_t N, int64_t V, uint64_t *__re
     if (bad)
         atomicOr(&sc->flags, kFlagIdRange);
     __syncthreads();
-    for (int k = 2; k <= kSortTile; k <<= 1) {
-        for (int j = k >> 1; j > 0; j >>= 1) {
+    for (int lk = 1; (1 << lk) <= kSortTile; ++lk) {
+        for (int lj = lk - 1; lj >= 0; --lj) {
+            const int j = 1 << lj;
 #pragma unroll
             for (int q = 0; q < kSortTile / 2 / kSortThreads; ++q) {
                 const int p = threadIdx.x + q * kSortThreads;  // pair index
-                const int i = (p / j) * 2 * j + (p % j);
+                const int i = ((p >> lj) << (lj + 1)) | (p & (j - 1));
                 const int l = i + j;
-                const bool up = (i & k) == 0;
+                const bool up = ((i >> lk) & 1) == 0;
                 const uint64_t a = s[i], b = s[l];
                 if ((a > b) == up) {
                     s[i] = b;
@@ -186,7 +187,7 @@ k_sp_heads(const uint64_t *__restrict__ sorted, int64_t N, int64_t V, int32_t *_
 }
 
 // Distinct ids and their runs.  Thread t of tile b owns sorted positions
-// 4096 b + 4 t .. + 3; an exclusive scan of run heads numbers the ids.
+// kSortTile b + 4 t .. + 3; an exclusive scan of run heads numbers the ids.
 __global__ void __launch_bounds__(kSortThreads)
 k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
               const int32_t *__restrict__ tilecnt, int32_t *__restrict__ uniq,
@@ -275,7 +276,7 @@ k_sp_chunks(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             float *__restrict__ carry, float *__restrict__ colpart, int D, int NS)
 {
     using F = typename Vec<VEC>::F;
-    constexpr int R = 8;
+    constexpr int R = 16;
     constexpr int kWarps = kThreads / 32;
     __shared__ float rp[kChunk][kWarps];
     __shared__ int fin[kChunk];
@@ -405,12 +406,21 @@ k_sp_carry(const int32_t *__restrict__ segoff, const DevScalars *__restrict__ sc
         float ps = 0.f;
         if (active) {
             const int64_t off = (int64_t)col * VEC;
+            // pieces in chunk order: the end piece of chunk q0, then the start
+            // pieces of q0+1 .. q1, eight loads in flight at a time
             F acc = load_g<VEC>(carry + ((int64_t)2 * q0 + 1) * D + off);
-            for (int q = q0 + 1; q <= q1; ++q) {
-                const F v = load_g<VEC>(carry + ((int64_t)2 * q) * D + off);
+            constexpr int kB = 8;
+            for (int qb = q0 + 1; qb <= q1; qb += kB) {
+                F v[kB];
 #pragma unroll
-                for (int e = 0; e < VEC; ++e)
-                    set_comp(acc, e, comp(acc, e) + comp(v, e));
+                for (int k = 0; k < kB; ++k)
+                    v[k] = (qb + k <= q1) ? load_g<VEC>(carry + ((int64_t)2 * (qb + k)) * D + off)
+                                          : zero_vec<VEC>();
+#pragma unroll
+                for (int k = 0; k < kB; ++k)
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e)
+                        set_comp(acc, e, comp(acc, e) + comp(v[k], e));
             }
             *reinterpret_cast<F *>(S + (int64_t)u * D + off) = acc;
 #pragma unroll
@@ -450,7 +460,7 @@ k_sp_vpass(float *__restrict__ r, int32_t *__restrict__ slot, const float *__res
            int NS, int64_t V, int D, double beta2, double one_minus_beta2,
            double *__restrict__ rsum_part)
 {
-    __shared__ double sh[kThreads];
+    __shared__ double sh[kThreads / 32];
     double rsum = 0.0;
     for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < V;
          i += (int64_t)gridDim.x * kThreads) {
@@ -468,11 +478,15 @@ k_sp_vpass(float *__restrict__ r, int32_t *__restrict__ slot, const float *__res
         r[i] = rn;
         rsum += (double)rn;
     }
-    sh[threadIdx.x] = rsum;
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+    if ((threadIdx.x & 31) == 0)
+        sh[threadIdx.x >> 5] = rsum;
     __syncthreads();
     if (threadIdx.x == 0) {
         double s = 0.0;
-        for (int k = 0; k < kThreads; ++k)
+        for (int k = 0; k < kThreads / 32; ++k)
             s += sh[k];
         rsum_part[blockIdx.x] = s;
     }
@@ -617,7 +631,7 @@ __global__ void k_sp_export(const int32_t *__restrict__ uniq, const int32_t *__r
 template <int VEC, int CPT>
 cudaError_t launch_sparse_t(const SparseArgs &a)
 {
-    constexpr int R = (4 / CPT) < 1 ? 1 : (4 / CPT);
+    constexpr int R = (8 / CPT) < 1 ? 1 : (8 / CPT);
     unsigned char *ws = a.ws;
     const Layout &L = a.lay;
     DevScalars *sc = reinterpret_cast<DevScalars *>(ws + L.scalars);

@@ -112,7 +112,9 @@ def test_sparse_parity_hyperparameters(cuda_device, opt):
 
 
 def test_sparse_equals_dense_on_scatter_summed_gradient(cuda_device):
-    """Section 2.2: the sparse step is the dense step on the summed rows."""
+    """Section 2.2: the sparse step is the dense step on the summed rows.
+    Gated like the oracle comparisons: each step both paths start from the
+    sparse path's W and state."""
     V, D, N = 3000, 512, 10000
     es, ed = make(V, D, "bf16", N), make(V, D, "bf16", 0)
     W0 = (torch.randn(V, D, device=cuda_device) * 0.02).to(torch.bfloat16)
@@ -121,6 +123,8 @@ def test_sparse_equals_dense_on_scatter_summed_gradient(cuda_device):
         ids, rows = batch(V, D, N, t, cuda_device, seed=9)
         G = torch.zeros(V, D, device=cuda_device, dtype=torch.float64)
         G.index_add_(0, ids, rows.double())
+        Wd.copy_(Ws)
+        ed.state.copy_(es.state)
         es.step_sparse(Ws, ids, rows, 1e-3, t)
         ed.step_dense(Wd, G.float(), 1e-3, t)
         torch.cuda.synchronize()
