@@ -64,8 +64,18 @@ def sparse_bytes(wl, U):
     return 4 * N * D + 8 * N + min(8 * U * D, 4 * N * D) + 2 * w * U * D + 8 * V + 8 * D
 
 
-SPARSE_KERNELS = ("tile_sort", "rank", "scatter", "heads", "segments", "chunks", "carry", "vpass",
+SPARSE_KERNELS = ("tile_sort", "rank", "scatter", "heads", "segments", "segsum", "carry", "vpass",
                   "state", "apply")
+TRACE_EVERY = 4  # every 4th timed step records kernel-boundary events
+
+
+def traced_steps(steps):
+    """Timed steps that record kernel boundaries: every TRACE_EVERY-th one,
+    and never all of them (at least one untraced step times the whole step)."""
+    if steps < 2:
+        raise SystemExit("--steps must be at least 2")
+    t = [k for k in range(steps) if k % TRACE_EVERY == TRACE_EVERY - 1]
+    return t or [steps - 1]
 
 
 def run_sparse(wl, dev, steps, warmup, flush, seed=0):
@@ -80,31 +90,40 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
     nk = len(SPARSE_KERNELS)
     t = 0
     warm = [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)]
-    for _ in range(warmup):
+    for i in range(warmup):
         t += 1
         flush.zero_()
-        emb.trace(warm)
+        emb.trace(warm if i % 2 else [])
         emb.step_sparse(W, ids, rows, wl.lr, t)
     torch.cuda.synchronize()
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for _ in range(steps)]
+    # untraced steps time the whole step (kernels overlap their launches);
+    # every TRACE_EVERY-th step records kernel boundaries instead
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(steps)]
+    traced = traced_steps(steps)
+    kern_ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for k in traced}
     for k in range(steps):
         t += 1
         flush.zero_()
-        emb.trace(events[k])
+        emb.trace(kern_ev.get(k, []))
+        step_ev[k][0].record()
         emb.step_sparse(W, ids, rows, wl.lr, t)
+        step_ev[k][1].record()
     torch.cuda.synchronize()
     emb.trace([])
     if emb.device_status() != 0:
         raise SystemExit("device status after the sparse steps")
-    per = {name: sum(ev[i].elapsed_time(ev[i + 1]) for ev in events) / steps
+    plain = [k for k in range(steps) if k not in kern_ev]
+    per = {name: sum(kern_ev[k][i].elapsed_time(kern_ev[k][i + 1]) for k in traced) / len(traced)
            for i, name in enumerate(SPARSE_KERNELS)}
-    ms = sum(ev[0].elapsed_time(ev[nk]) for ev in events) / steps
+    ms = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain)
+    ms_traced = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in traced) / len(traced)
     B = sparse_bytes(wl, U)
     return {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "unique_ids": U,
             "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
             "algorithmic_bytes": B, "touched_params_per_s": U * wl.D / (ms * 1e-3),
             "occurrence_params_per_s": wl.N * wl.D / (ms * 1e-3),
-            "kernels_ms": per, "gpu_launches": nk * steps}
+            "kernels_ms": per, "ms_per_step_traced": ms_traced, "gpu_launches": nk * steps}
 
 
 def measured_hbm_peak():
@@ -248,7 +267,7 @@ def sparse_kernel_bytes(wl, U):
     """Algorithmic bytes per launch of the segment-sum kernel (grad rows read,
     summed rows written, sorted order read) and of the apply kernel."""
     N, D, w = wl.N, wl.D, wbytes(wl)
-    return {"chunks": 4 * N * D + 4 * U * D + 8 * N, "apply": 4 * U * D + 2 * w * U * D + 8 * U}
+    return {"segsum": 4 * N * D + 4 * U * D + 8 * N, "apply": 4 * U * D + 2 * w * U * D + 8 * U}
 
 
 def run_sparse_line(args, wl, world, rank, dev):
@@ -261,7 +280,7 @@ def run_sparse_line(args, wl, world, rank, dev):
     ms = allreduce_max(world, sp["ms_per_step"])
     peak, peak_kind = measured_hbm_peak()
     kb = sparse_kernel_bytes(wl, sp["unique_ids"])
-    ach = kb["chunks"] / (sp["kernels_ms"]["chunks"] * 1e-3) / 1e9
+    ach = kb["segsum"] / (sp["kernels_ms"]["segsum"] * 1e-3) / 1e9
     line = {
         "metric": METRIC, "value": world * sp["algorithmic_bytes"] / (ms * 1e-3) / 1e9, "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
@@ -270,9 +289,9 @@ def run_sparse_line(args, wl, world, rank, dev):
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "w_dtype": wl.wdtype,
                    "ids": "int64", "l2": "flushed between steps (512 MiB write, outside the events)",
                    "parallelism": f"replicas x{world}"},
-        "roofline": {"bound": "hbm", "kernel": "k_sp_chunks", "achieved": ach, "peak": peak,
+        "roofline": {"bound": "hbm", "kernel": "k_sp_segsum", "achieved": ach, "peak": peak,
                      "unit": "GB/s", "frac": ach / peak, "peak_kind": peak_kind, "traffic": None,
-                     "algorithmic_bytes_per_launch": kb["chunks"]},
+                     "algorithmic_bytes_per_launch": kb["segsum"]},
         "cpu_baseline": None, "e2e": None, "gpu_launches": sp["gpu_launches"],
         "clocks": clocks.summary(), "sparse": sp,
     }
@@ -303,14 +322,20 @@ def run_ours(args, world, rank, local):
         emb.step_dense(W, G, wl.lr, t)
 
     warm_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    # warm-up alternates traced and untraced steps
     t = 0
-    for _ in range(args.warmup):
+    for i in range(args.warmup):
         t += 1
         flush.zero_()
-        one_step(t, warm_ev)
+        one_step(t, warm_ev if i % 2 else [])
     torch.cuda.synchronize()
 
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    # untraced steps time the whole step (kernels overlap their launches);
+    # every TRACE_EVERY-th step records kernel boundaries instead
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.steps)]
+    traced = traced_steps(args.steps)
+    events = {k: [torch.cuda.Event(enable_timing=True) for _ in range(4)] for k in traced}
     barrier(world)
     torch.cuda.synchronize()
     wall0 = time.perf_counter()
@@ -318,7 +343,10 @@ def run_ours(args, world, rank, local):
         for k in range(args.steps):
             t += 1
             flush.zero_()
-            one_step(t, events[k])
+            emb.trace(events.get(k, []))
+            step_ev[k][0].record(stream)
+            emb.step_dense(W, G, wl.lr, t)
+            step_ev[k][1].record(stream)
         torch.cuda.synchronize()
         barrier(world)
     wall = time.perf_counter() - wall0
@@ -327,14 +355,15 @@ def run_ours(args, world, rank, local):
     if status != 0:
         raise SystemExit(f"device status {status} after the timed steps")
 
-    per = {"reduce": [], "state": [], "apply": [], "step": []}
-    for ev in events:
+    per = {"reduce": [], "state": [], "apply": [], "traced_step": []}
+    for ev in events.values():
         per["reduce"].append(ev[0].elapsed_time(ev[1]))
         per["state"].append(ev[1].elapsed_time(ev[2]))
         per["apply"].append(ev[2].elapsed_time(ev[3]))
-        per["step"].append(ev[0].elapsed_time(ev[3]))
+        per["traced_step"].append(ev[0].elapsed_time(ev[3]))
     mean = {k: sum(v) / len(v) for k, v in per.items()}
-    ms = allreduce_max(world, mean["step"])
+    plain = [k for k in range(args.steps) if k not in events]
+    ms = allreduce_max(world, sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain))
 
     B = step_bytes(wl)
     value = world * B / (ms * 1e-3) / 1e9
@@ -386,7 +415,8 @@ def run_ours(args, world, rank, local):
     sparse = None
     if not args.no_sparse:
         swl = synth.WORKLOADS["sparse_v262144_d2048_bf16_n32768"]
-        sparse = run_sparse(swl, dev, max(10, min(args.steps, 100)), args.warmup, flush, seed=rank)
+        sparse = run_sparse(swl, dev, max(2 * TRACE_EVERY, min(args.steps, 100)), args.warmup, flush,
+                            seed=rank)
         sparse["frac_of_nominal_8TBs"] = sparse["value"] / NOMINAL_HBM_GBS
         sparse["frac_of_measured_hbm"] = sparse["value"] / peak
 
@@ -406,6 +436,8 @@ def run_ours(args, world, rank, local):
         "frac_of_nominal_8TBs": value / world / NOMINAL_HBM_GBS,
         "frac_of_measured_hbm": value / world / peak,
         "kernels": kern,
+        "ms_per_step_traced": mean["traced_step"],
+        "timing": f"step time: CUDA events around each untraced step; kernel times: every {TRACE_EVERY}th step records events at kernel boundaries",
         "wall_s_timed_region": wall,
         "sparse": sparse,
     }

@@ -7,6 +7,7 @@ this runs on a machine without a GPU too.
 import concurrent.futures
 import os
 import subprocess
+import tempfile
 
 PKG = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(PKG)
@@ -31,8 +32,8 @@ def _deps():
         [os.path.join(INCLUDE, f) for f in os.listdir(INCLUDE) if f.endswith(".h")]
 
 
-def _compile(src, extra):
-    obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
+def _compile(src, extra, objdir):
+    obj = os.path.join(objdir, os.path.basename(src)[:-3] + ".o")
     subprocess.run([NVCC, *ARCH, *FLAGS, *extra, "-c", src, "-o", obj], check=True)
     return obj
 
@@ -45,11 +46,13 @@ def build_library(force: bool = False, verbose_ptxas: bool = False) -> str:
     os.makedirs(BUILD, exist_ok=True)
     os.makedirs(LIB_DIR, exist_ok=True)
     extra = ["-Xptxas", "-v"] if verbose_ptxas else []
-    with concurrent.futures.ThreadPoolExecutor(max_workers=len(sources())) as ex:
-        objs = list(ex.map(lambda s: _compile(s, extra), sources()))
-    tmp = LIB + f".tmp{os.getpid()}"
-    subprocess.run([NVCC, *ARCH, "-shared", "-o", tmp, *objs], check=True)
-    os.replace(tmp, LIB)
+    # objects of concurrent builds (parallel test workers) never collide
+    with tempfile.TemporaryDirectory(dir=BUILD) as objdir:
+        with concurrent.futures.ThreadPoolExecutor(max_workers=len(sources())) as ex:
+            objs = list(ex.map(lambda s: _compile(s, extra, objdir), sources()))
+        tmp = LIB + f".tmp{os.getpid()}"
+        subprocess.run([NVCC, *ARCH, "-shared", "-o", tmp, *objs], check=True)
+        os.replace(tmp, LIB)
     return LIB
 
 

@@ -31,7 +31,6 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
         const size_t N = (size_t)max_sparse_N;
         const size_t Npad = (N + kSortTile - 1) / kSortTile * kSortTile;
         const size_t nslices = (size_t)((D + kThreads - 1) / kThreads);
-        const size_t nchunks = (N + kChunk - 1) / kChunk;
         L.sp_keys = take(sizeof(uint64_t) * Npad);
         L.sp_rank = take(sizeof(int32_t) * Npad);
         L.sp_sorted = take(sizeof(uint64_t) * N);
@@ -42,7 +41,8 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
         L.sp_segoff = take(sizeof(int32_t) * (N + 1));
         L.sp_slot = take(sizeof(int32_t) * (size_t)V);
         L.sp_rowpart = take(sizeof(float) * N * nslices);
-        L.sp_carry = take(sizeof(float) * 2 * nchunks * (size_t)D);
+        L.sp_carry = take(sizeof(float) * 2 * (size_t)kGridCtas * (size_t)D);
+        L.sp_bounds = take(sizeof(int32_t) * ((size_t)kGridCtas + 1));
         L.sp_rows = take(sizeof(float) * N * (size_t)D);
     }
     L.total = off;

@@ -60,6 +60,9 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
     const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
 
+    grid_dep_wait();    // the first kernel of a step: returns at once
+    grid_dep_launch();  // the state pass may start launching now; it waits for this grid
+
     // per-warp row sums of up to kRowBuf rows, finalised together
     constexpr int kRowBuf = 128;
     __shared__ float red[kWarps][kRowBuf];
@@ -207,6 +210,8 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
     const int j = blockIdx.x * kStateCols + lane;
     __shared__ double part[kW][32];
     __shared__ bool am_last;
+    grid_dep_wait();  // column partials and row sums of the reduce pass
+    grid_dep_launch();
 
     // rows w, w + 8, w + 16, ...: sixteen loads in flight, summed pairwise
     // in fp32 within the batch and in fp64 across batches
@@ -301,6 +306,26 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
     const int64_t step = (int64_t)rg * R;
     const int64_t nblocks = (row1 - row0 + step - 1) / step;
 
+    // While the state pass finishes: pull this thread's first rows of G and
+    // W (the last iteration block, walked first) towards L2.
+    if (nblocks > 0) {
+        const int64_t base = row0 + (nblocks - 1) * step;
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+            for (int cc = 0; cc < CPT; ++cc) {
+                const int col = l + cc * tpr;
+                if (i < row1 && col < DV) {
+                    const int64_t idx = i * D + (int64_t)col * VEC;
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(G + idx));
+                    asm volatile("prefetch.global.L2 [%0];" ::"l"(static_cast<const char *>(W) +
+                                                                   idx * (BF16 ? 2 : 4)));
+                }
+            }
+        }
+    }
+    grid_dep_wait();  // c, s (state pass) and r (reduce pass)
+    grid_dep_launch();
+
     // column scale sqrt(chat_j / s) (FULL), sqrt(chat_j) (COL) or 1 (ROW)
     const float inv_s = (variant == EMBER_VARIANT_FULL) ? sc->inv_s : 1.f;
     for (int j = tid; j < D; j += kThreads)
@@ -362,23 +387,36 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     const int rg = kThreads / a.map.tpr;
     const size_t shmem = (rg > 1) ? (size_t)D * sizeof(float) : 0;
 
+    // With tracing, events sit between the kernels and each launch simply
+    // follows the previous one; without, kernels 2 and 3 use programmatic
+    // dependent launch.
+    const bool pdl = (a.trace == nullptr);
+    cudaError_t e;
     if (a.trace)
         cudaEventRecord(a.trace[0], a.stream);
-    k_reduce_dense<VEC, CPT, R1><<<nparts, kThreads, shmem, a.stream>>>(
-        a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2);
+    e = launch_k(k_reduce_dense<VEC, CPT, R1>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
+                 a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2);
+    if (e != cudaSuccess)
+        return e;
     if (a.trace)
         cudaEventRecord(a.trace[1], a.stream);
-    launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                 a.one_minus_beta2, a.inv_bc, a.stream);
+    e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                     a.one_minus_beta2, a.inv_bc, a.stream, pdl);
+    if (e != cudaSuccess)
+        return e;
     if (a.trace)
         cudaEventRecord(a.trace[2], a.stream);
     const size_t cs_bytes = (size_t)D * sizeof(float);
     if (a.wbf16)
-        k_apply_dense<VEC, CPT, R3, true><<<nparts, kThreads, cs_bytes, a.stream>>>(
-            a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+        e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
+                     a.stream, pdl, a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
+                     a.eps, a.lr_signed, a.variant);
     else
-        k_apply_dense<VEC, CPT, R3, false><<<nparts, kThreads, cs_bytes, a.stream>>>(
-            a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+        e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
+                     a.stream, pdl, a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
+                     a.eps, a.lr_signed, a.variant);
+    if (e != cudaSuccess)
+        return e;
     if (a.trace)
         cudaEventRecord(a.trace[3], a.stream);
     return cudaGetLastError();
@@ -386,13 +424,13 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 
 }  // namespace
 
-void launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum, float *c,
-                  double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                  double one_minus_beta2, double inv_bc, cudaStream_t stream)
+cudaError_t launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum,
+                         float *c, double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl)
 {
     const int nstate = (D + kStateCols - 1) / kStateCols;
-    k_state_dense<<<nstate, kStateThreads, 0, stream>>>(colpart, nparts, rsum_part, nrsum, c, csum_part,
-                                                        sc, V, D, beta2, one_minus_beta2, inv_bc);
+    return launch_k(k_state_dense, dim3(nstate), dim3(kStateThreads), 0, stream, pdl, colpart, nparts,
+                    rsum_part, nrsum, c, csum_part, sc, V, D, beta2, one_minus_beta2, inv_bc);
 }
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)

@@ -9,6 +9,12 @@
 namespace ember {
 namespace dev {
 
+// Programmatic dependent launch: wait until the kernels this one depends on
+// have completed and their writes are visible (a no-op when launched
+// without the attribute), and allow the next kernel to start launching.
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;"); }
+
 template <int VEC> struct Vec;
 template <> struct Vec<4> { using F = float4; };
 template <> struct Vec<1> { using F = float; };

@@ -42,10 +42,9 @@ struct DevScalars {
 };
 
 // Sparse step: ids are sorted in tiles of kSortTile keys by kSortThreads
-// threads; the sorted occurrences are summed in chunks of kChunk.
+// threads.
 constexpr int kSortTile = 1024;
 constexpr int kSortThreads = 256;
-constexpr int kChunk = 32;
 
 // Workspace layout (byte offsets, each 256-byte aligned).
 struct Layout {
@@ -65,7 +64,8 @@ struct Layout {
     size_t sp_segoff;   // int32[N + 1]  first sorted position of each distinct id
     size_t sp_slot;     // int32[V]      1 + distinct-id index of a touched row, else 0
     size_t sp_rowpart;  // float[N * ceil(D / kThreads)]  sum g^2 per (distinct id, slice)
-    size_t sp_carry;    // float[2 * ceil(N / kChunk) * D]  partial sums of cut segments
+    size_t sp_carry;    // float[2 * kGridCtas * D]  partial sums of runs cut by worker ranges
+    size_t sp_bounds;   // int32[kGridCtas + 1]  first sorted position of each worker range
     size_t sp_rows;     // float[N * D]  summed gradient row of each distinct id
     size_t total;
 };
@@ -102,9 +102,9 @@ struct DenseArgs {
 
 cudaError_t launch_dense_step(const DenseArgs &a);
 
-void launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum, float *c,
-                  double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                  double one_minus_beta2, double inv_bc, cudaStream_t stream);
+cudaError_t launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum,
+                         float *c, double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl);
 
 struct SparseArgs {
     int64_t V, D, N;
@@ -134,6 +134,27 @@ cudaError_t launch_sparse_unique(const SparseArgs &a, int32_t *uniq_out, int32_t
                                  int32_t *n_unique_out);
 
 constexpr int kMaxTraceEvents = 16;
+
+// Launch `kernel` on `stream`.  With pdl = true the launch may begin while
+// the previous kernel on the stream is still finishing (programmatic
+// dependent launch); every kernel launched this way calls grid_dep_wait()
+// before it reads anything an earlier kernel wrote.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_k(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                     cudaStream_t stream, bool pdl, Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = pdl ? attr : nullptr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kernel, static_cast<KArgs>(args)...);
+}
 
 }  // namespace ember
 

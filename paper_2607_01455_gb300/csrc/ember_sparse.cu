@@ -21,18 +21,21 @@
 //   dedup     k_sp_heads, k_sp_segments: run heads, the distinct ids
 //             (ascending), where each id's run starts, and a V-entry map from
 //             a touched row to its distinct-id index.
-//   segsum    k_sp_chunks, k_sp_carry: the summed gradient row of every
+//   segsum    k_sp_segsum, k_sp_carry: the summed gradient row of every
 //             distinct id, adding its occurrences in increasing occurrence
 //             order; per (id, column slice) sums of g^2; per-CTA column sums
-//             of g^2.  The sorted occurrences are cut into chunks of 32 so the
-//             work is even however skewed the id counts are (a Zipf head id
-//             can own thousands of occurrences); a run that crosses chunk
-//             boundaries is summed piecewise and its pieces are added in
-//             chunk order by k_sp_carry.
+//             of g^2.  Each worker owns a contiguous, equal share of the
+//             sorted occurrences, so the work is even however skewed the id
+//             counts are (a Zipf head id can own thousands of occurrences);
+//             a run that crosses worker boundaries leaves one piece per
+//             worker, which k_sp_carry adds in worker order.
 //   rows      k_sp_vpass: r for all V rows, the sums of new r per CTA, and the
 //             touched-row map cleared for the next step.
 //   state     the dense step's column/normaliser pass.
 //   apply     k_sp_apply: the update of the touched rows only.
+//
+// Every kernel after the first is launched with programmatic dependent
+// launch and waits (griddepcontrol.wait) before it reads earlier results.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -55,6 +58,8 @@ k_sp_tile_sort(const IdT *__restrict__ ids, int64_t N, int64_t V, uint64_t *__re
     __shared__ uint64_t s[kSortTile];
     const int64_t base = (int64_t)blockIdx.x * kSortTile;
     bool bad = false;
+    grid_dep_wait();  // first kernel of a step: returns at once
+    grid_dep_launch();
 #pragma unroll
     for (int q = 0; q < kKeysPerThread; ++q) {
         const int i = threadIdx.x + q * kSortThreads;
@@ -105,6 +110,8 @@ __global__ void __launch_bounds__(kSortThreads)
 k_sp_rank(const uint64_t *__restrict__ keys, int32_t *__restrict__ rank)
 {
     const int own = blockIdx.x, other = blockIdx.y;
+    grid_dep_wait();  // tile-sorted keys
+    grid_dep_launch();
     if (own == other)
         return;
     __shared__ uint64_t s[kSortTile];
@@ -136,6 +143,8 @@ k_sp_rank(const uint64_t *__restrict__ keys, int32_t *__restrict__ rank)
 __global__ void k_sp_scatter(const uint64_t *__restrict__ keys, const int32_t *__restrict__ rank,
                              int64_t npad, uint64_t *__restrict__ sorted)
 {
+    grid_dep_wait();  // ranks
+    grid_dep_launch();
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < npad;
          q += (int64_t)gridDim.x * blockDim.x) {
         const uint64_t x = keys[q];
@@ -165,6 +174,8 @@ __global__ void __launch_bounds__(kSortThreads)
 k_sp_heads(const uint64_t *__restrict__ sorted, int64_t N, int64_t V, int32_t *__restrict__ tilecnt)
 {
     __shared__ int sh[kSortThreads / 32];
+    grid_dep_wait();  // sorted keys
+    grid_dep_launch();
     const int64_t p0 = (int64_t)blockIdx.x * kSortTile + (int64_t)threadIdx.x * kKeysPerThread;
     int nh = 0, nv = 0;
 #pragma unroll
@@ -197,6 +208,8 @@ k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
     __shared__ int pre[2];
     __shared__ int wsum[kSortThreads / 32];
     __shared__ int sh[kSortThreads / 32];
+    grid_dep_wait();  // per-tile counts
+    grid_dep_launch();
     if (threadIdx.x == 0) {
         int a = 0, b = 0;
         for (int t = 0; t < (int)blockIdx.x; ++t) {
@@ -266,20 +279,80 @@ k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
     }
 }
 
+// Workers split the sorted occurrences into contiguous ranges of equal
+// cost, cost(p) = p + segidx[p]: one unit per occurrence row read and one
+// per summed row written (runs are numbered in order, so the cost rises by
+// one or two per position).  Worker w owns [first(w), first(w + 1)), where
+// first(w) is the smallest position whose cost reaches T(w) = w C / nw and
+// C = n_valid + U.
+__device__ __forceinline__ int64_t cost_target(int w, int nw, int64_t C)
+{
+    return ((int64_t)w * C) / nw;
+}
+
+// Smallest p in [0, n_valid] with p + segidx[p] >= T (position n_valid
+// counts as reaching every target).  Block-wide 256-way search: each round
+// probes kThreads evenly spaced positions and keeps the one interval that
+// holds the answer.
+__device__ int block_first_reaching(const int32_t *__restrict__ segidx, int n_valid, int64_t T)
+{
+    __shared__ int lo_hi[2];
+    int lo = 0, hi = n_valid;  // answer in [lo, hi]
+    while (lo < hi) {
+        const int64_t len = hi - lo;
+        const int t = threadIdx.x;
+        const int p = lo + (int)((len * t) / kThreads);
+        const bool reached = (int64_t)p + segidx[p] >= T;  // p < hi <= n_valid
+        const int below = __syncthreads_count(!reached);  // probes before the answer
+        if (t == 0) {
+            int nlo = lo, nhi = hi;
+            if (below > 0)
+                nlo = lo + (int)((len * (below - 1)) / kThreads) + 1;
+            if (below < kThreads)
+                nhi = lo + (int)((len * below) / kThreads);
+            lo_hi[0] = nlo;
+            lo_hi[1] = nhi;
+        }
+        __syncthreads();
+        lo = lo_hi[0];
+        hi = lo_hi[1];
+        __syncthreads();
+    }
+    return lo;
+}
+
+// Worker whose range holds sorted position p of run u.
+__device__ __forceinline__ int worker_of(int p, int u, int nw, int64_t C)
+{
+    const int64_t c = (int64_t)p + u;
+    int w = (int)((c * nw) / C);
+    while (w + 1 < nw && cost_target(w + 1, nw, C) <= c)
+        ++w;
+    while (w > 0 && cost_target(w, nw, C) > c)
+        --w;
+    return w;
+}
+
 // Sum the occurrences of each run.  CTA b works on column slice b % NS
-// (kThreads vector columns) of chunks b / NS, b / NS + nw, ...
+// (kThreads vector columns) of the sorted positions of worker b / NS, adding
+// each run's rows in increasing occurrence order with a running sum that
+// crosses the worker's whole range.  A run that starts before the range or
+// ends after it leaves its piece in the carry buffer (slot 0: the range's
+// first run, slot 1: its last run); k_sp_carry adds the pieces in worker
+// order.  Completed runs are written to S with their sum of g^2 per slice.
 template <int VEC>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
-k_sp_chunks(const float *__restrict__ rows, const int32_t *__restrict__ perm,
-            const int32_t *__restrict__ segidx, const int32_t *__restrict__ segoff,
-            const DevScalars *__restrict__ sc, float *__restrict__ S, float *__restrict__ rowpart,
-            float *__restrict__ carry, float *__restrict__ colpart, int D, int NS)
+k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
+            const int32_t *__restrict__ segidx, const DevScalars *__restrict__ sc,
+            float *__restrict__ S, float *__restrict__ rowpart, float *__restrict__ carry,
+            float *__restrict__ colpart, int32_t *__restrict__ bounds, int D, int NS)
 {
     using F = typename Vec<VEC>::F;
     constexpr int R = 16;
     constexpr int kWarps = kThreads / 32;
-    __shared__ float rp[kChunk][kWarps];
-    __shared__ int fin[kChunk];
+    constexpr int kFin = 32;  // completed runs buffered before their g^2 sums are written
+    __shared__ float rp[kFin][kWarps];
+    __shared__ int fin[kFin];
     const int DV = D / VEC;
     const int sigma = blockIdx.x % NS;
     const int w = blockIdx.x / NS;
@@ -287,22 +360,56 @@ k_sp_chunks(const float *__restrict__ rows, const int32_t *__restrict__ perm,
     const int col = sigma * kThreads + threadIdx.x;
     const bool active = col < DV;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    grid_dep_wait();  // runs and occurrence order from the dedup kernels
+    grid_dep_launch();
     const int n_valid = sc->n_valid;
-    const int nchunks = (n_valid + kChunk - 1) / kChunk;
     float colacc[VEC];
 #pragma unroll
     for (int e = 0; e < VEC; ++e)
         colacc[e] = 0.f;
 
-    for (int q = w; w < nw && q < nchunks; q += nw) {
-        const int p0 = q * kChunk;
-        const int p1 = min(p0 + kChunk, n_valid);
-        int nfin = 0;
-        int cur = segidx[p0];
+    const bool worker = w < nw && n_valid > 0;
+    int p0 = 0, p1 = 0;
+    if (worker) {
+        const int64_t C = (int64_t)n_valid + sc->n_unique;
+        p0 = block_first_reaching(segidx, n_valid, cost_target(w, nw, C));
+        p1 = (w + 1 == nw) ? n_valid : block_first_reaching(segidx, n_valid, cost_target(w + 1, nw, C));
+        if (sigma == 0 && threadIdx.x == 0) {
+            bounds[w] = p0;
+            if (w + 1 == nw)
+                bounds[nw] = n_valid;
+        }
+        if (p0 == p1 && active) {
+            // an empty range holds no piece of the run that spans it
+            const F z = zero_vec<VEC>();
+            *reinterpret_cast<F *>(carry + ((int64_t)2 * w) * D + (int64_t)col * VEC) = z;
+            *reinterpret_cast<F *>(carry + ((int64_t)2 * w + 1) * D + (int64_t)col * VEC) = z;
+        }
+    }
+    int nfin = 0;
+    auto drain = [&]() {  // uniform: all threads call it together
+        __syncthreads();
+        if (threadIdx.x < nfin) {
+            float t = 0.f;
+            for (int k = 0; k < kWarps; ++k)
+                t += rp[threadIdx.x][k];
+            rowpart[(int64_t)fin[threadIdx.x] * NS + sigma] = t;
+        }
+        __syncthreads();
+        nfin = 0;
+    };
+    if (p0 < p1) {
+        // Only the range's first run can have started before it and only
+        // its last run can continue after it; decide both once, here.
+        const int u_first = segidx[p0];
+        const int u_last = segidx[p1 - 1];
+        const bool first_cut = p0 > 0 && segidx[p0 - 1] == u_first;
+        const bool last_cut = p1 < n_valid && segidx[p1] == u_last;
+        int cur = u_first;
         F acc = zero_vec<VEC>();
         auto flush = [&](int u) {
-            const bool before = segoff[u] < p0;
-            const bool after = segoff[u + 1] > p1;
+            const bool before = first_cut && u == u_first;
+            const bool after = last_cut && u == u_last;
             if (!before && !after) {
                 float ps = 0.f;
                 if (active) {
@@ -322,9 +429,11 @@ k_sp_chunks(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                 if (threadIdx.x == 0)
                     fin[nfin] = u;
                 ++nfin;
+                if (nfin == kFin)
+                    drain();
             } else if (active) {
-                const int which = before ? 0 : 1;  // piece at the chunk's start / end
-                *reinterpret_cast<F *>(carry + ((int64_t)2 * q + which) * D + (int64_t)col * VEC) = acc;
+                const int which = before ? 0 : 1;
+                *reinterpret_cast<F *>(carry + ((int64_t)2 * w + which) * D + (int64_t)col * VEC) = acc;
             }
         };
         for (int pb = p0; pb < p1; pb += R) {
@@ -356,66 +465,74 @@ k_sp_chunks(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             }
         }
         flush(cur);
-        __syncthreads();
-        if (threadIdx.x < nfin) {
-            float s = 0.f;
-            for (int k = 0; k < kWarps; ++k)
-                s += rp[threadIdx.x][k];
-            rowpart[(int64_t)fin[threadIdx.x] * NS + sigma] = s;
-        }
-        __syncthreads();
     }
+    if (nfin > 0)
+        drain();
     float *out = colpart + (int64_t)blockIdx.x * D;
     for (int j = threadIdx.x; j < D; j += kThreads)
         out[j] = 0.f;
     __syncthreads();
-    if (active && w < nw)
+    if (active && worker)
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
             out[col * VEC + e] = colacc[e];
 }
 
-// Runs cut by chunk boundaries: add their pieces in chunk order.
+// Runs cut by worker boundaries.  CTA b handles boundary bd = b / NS + 1
+// (position first(bd)) on slice b % NS: if the run holding that position
+// started inside the previous worker's range, this CTA adds the run's
+// pieces -- the previous worker's last piece, then the first pieces of the
+// following workers up to the one holding the run's end -- in worker order.
 template <int VEC>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
-k_sp_carry(const int32_t *__restrict__ segoff, const DevScalars *__restrict__ sc,
+k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segoff,
+           const int32_t *__restrict__ bounds, const DevScalars *__restrict__ sc,
            const float *__restrict__ carry, float *__restrict__ S, float *__restrict__ rowpart,
-           float *__restrict__ colpart, int D, int NS)
+           float *__restrict__ colpart, int D, int NS, int nw)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
     __shared__ float red[kWarps];
     const int DV = D / VEC;
     const int sigma = blockIdx.x % NS;
-    const int w = blockIdx.x / NS;
-    const int nw = gridDim.x / NS;
+    const int bd = blockIdx.x / NS + 1;
     const int col = sigma * kThreads + threadIdx.x;
     const bool active = col < DV;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int U = sc->n_unique;
+    grid_dep_wait();  // carry pieces from k_sp_segsum
+    grid_dep_launch();
+    const int n_valid = sc->n_valid;
     float colacc[VEC];
 #pragma unroll
     for (int e = 0; e < VEC; ++e)
         colacc[e] = 0.f;
-
-    for (int u = w; w < nw && u < U; u += nw) {
-        const int s0 = segoff[u], s1 = segoff[u + 1];
-        const int q0 = s0 / kChunk, q1 = (s1 - 1) / kChunk;
-        if (q0 == q1)
-            continue;
+    bool mine = false;
+    int u = 0, w0 = 0, w1 = 0;
+    if (bd < nw && n_valid > 0) {
+        const int p = bounds[bd];
+        if (p < n_valid) {
+            u = segidx[p];
+            const int s0 = segoff[u], s1 = segoff[u + 1];
+            w0 = bd - 1;
+            mine = s0 < p && s0 >= bounds[w0];
+            const int64_t C = (int64_t)n_valid + sc->n_unique;
+            w1 = worker_of(s1 - 1, u, nw, C);
+        }
+    }
+    if (mine) {
         float ps = 0.f;
         if (active) {
             const int64_t off = (int64_t)col * VEC;
-            // pieces in chunk order: the end piece of chunk q0, then the start
-            // pieces of q0+1 .. q1, eight loads in flight at a time
-            F acc = load_g<VEC>(carry + ((int64_t)2 * q0 + 1) * D + off);
+            F acc = load_g<VEC>(carry + ((int64_t)2 * w0 + 1) * D + off);
             constexpr int kB = 8;
-            for (int qb = q0 + 1; qb <= q1; qb += kB) {
+            for (int qb = w0 + 1; qb <= w1; qb += kB) {
                 F v[kB];
 #pragma unroll
-                for (int k = 0; k < kB; ++k)
-                    v[k] = (qb + k <= q1) ? load_g<VEC>(carry + ((int64_t)2 * (qb + k)) * D + off)
-                                          : zero_vec<VEC>();
+                for (int k = 0; k < kB; ++k) {
+                    // workers with an empty range wrote zero pieces
+                    const int q = qb + k;
+                    v[k] = (q <= w1) ? load_g<VEC>(carry + ((int64_t)2 * q) * D + off) : zero_vec<VEC>();
+                }
 #pragma unroll
                 for (int k = 0; k < kB; ++k)
 #pragma unroll
@@ -437,18 +554,17 @@ k_sp_carry(const int32_t *__restrict__ segoff, const DevScalars *__restrict__ sc
             red[warp] = ps;
         __syncthreads();
         if (threadIdx.x == 0) {
-            float s = 0.f;
+            float t = 0.f;
             for (int k = 0; k < kWarps; ++k)
-                s += red[k];
-            rowpart[(int64_t)u * NS + sigma] = s;
+                t += red[k];
+            rowpart[(int64_t)u * NS + sigma] = t;
         }
-        __syncthreads();
     }
     float *out = colpart + (int64_t)blockIdx.x * D;
     for (int j = threadIdx.x; j < D; j += kThreads)
         out[j] = 0.f;
     __syncthreads();
-    if (active && w < nw)
+    if (active && mine)
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
             out[col * VEC + e] = colacc[e];
@@ -461,6 +577,8 @@ k_sp_vpass(float *__restrict__ r, int32_t *__restrict__ slot, const float *__res
            double *__restrict__ rsum_part)
 {
     __shared__ double sh[kThreads / 32];
+    grid_dep_wait();  // per-run sums of g^2
+    grid_dep_launch();
     double rsum = 0.0;
     for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < V;
          i += (int64_t)gridDim.x * kThreads) {
@@ -508,6 +626,8 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__r
     const int rg = kThreads / tpr;
     const int g = tid / tpr;
     const int l = tid - g * tpr;
+    grid_dep_wait();  // s, c, r and the summed rows
+    grid_dep_launch();
     const int U = sc->n_unique;
     const float inv_s = (variant == EMBER_VARIANT_FULL) ? sc->inv_s : 1.f;
     for (int j = tid; j < D; j += kThreads)
@@ -515,22 +635,33 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__r
     __syncthreads();
 
     const int64_t stride = (int64_t)gridDim.x * rg * R;
-    for (int64_t ub = ((int64_t)blockIdx.x * rg + g) * R; ub < U; ub += stride) {
+    const int64_t ub0 = ((int64_t)blockIdx.x * rg + g) * R;
+    // row ids of the next iteration are loaded while this one's rows are in flight
+    int64_t next[R];
+#pragma unroll
+    for (int k = 0; k < R; ++k)
+        next[k] = (ub0 + k < U) ? (int64_t)uniq[ub0 + k] : -1;
+    for (int64_t ub = ub0; ub < U; ub += stride) {
         F gv[R][CPT];
         WT wr[R][CPT];
         int64_t row[R];
 #pragma unroll
         for (int k = 0; k < R; ++k) {
             const int64_t u = ub + k;
-            row[k] = (u < U) ? (int64_t)uniq[u] : -1;
+            row[k] = next[k];
 #pragma unroll
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
-                if (u < U && col < DV) {
+                if (row[k] >= 0 && col < DV) {
                     gv[k][cc] = load_g<VEC>(S + u * D + (int64_t)col * VEC);
                     wr[k][cc] = load_w<BF16, VEC>(W, row[k] * D + (int64_t)col * VEC);
                 }
             }
+        }
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t un = ub + stride + k;
+            next[k] = (un < U) ? (int64_t)uniq[un] : -1;
         }
 #pragma unroll
         for (int k = 0; k < R; ++k) {
@@ -560,11 +691,20 @@ struct Tracer {
     const cudaEvent_t *ev;
     int n, next;
     cudaStream_t s;
+    bool launched = false;  // a kernel of this step is already on the stream
     void mark()
     {
         if (ev && next < n)
             cudaEventRecord(ev[next], s);
         ++next;
+    }
+    // programmatic dependent launch for every kernel after the first,
+    // unless events are recorded between the kernels
+    bool pdl()
+    {
+        const bool p = launched && ev == nullptr;
+        launched = true;
+        return p;
     }
 };
 
@@ -587,27 +727,28 @@ void launch_sort_dedup(const SparseArgs &a, Tracer &tr)
         const int T = (int)((a.N + kSortTile - 1) / kSortTile);
         const int64_t npad = (int64_t)T * kSortTile;
         if (a.ids64)
-            k_sp_tile_sort<int64_t><<<T, kSortThreads, 0, a.stream>>>(
-                static_cast<const int64_t *>(a.ids), a.N, a.V, keys, rank, sc);
+            launch_k(k_sp_tile_sort<int64_t>, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(),
+                     static_cast<const int64_t *>(a.ids), a.N, a.V, keys, rank, sc);
         else
-            k_sp_tile_sort<int32_t><<<T, kSortThreads, 0, a.stream>>>(
-                static_cast<const int32_t *>(a.ids), a.N, a.V, keys, rank, sc);
+            launch_k(k_sp_tile_sort<int32_t>, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(),
+                     static_cast<const int32_t *>(a.ids), a.N, a.V, keys, rank, sc);
         tr.mark();
         if (T > 1) {
-            k_sp_rank<<<dim3(T, T), kSortThreads, 0, a.stream>>>(keys, rank);
+            launch_k(k_sp_rank, dim3(T, T), dim3(kSortThreads), 0, a.stream, tr.pdl(), keys, rank);
             tr.mark();
         }
         const int nsc = (int)((npad + kThreads - 1) / kThreads);
-        k_sp_scatter<<<nsc, kThreads, 0, a.stream>>>(keys, rank, npad, sorted);
+        launch_k(k_sp_scatter, dim3(nsc), dim3(kThreads), 0, a.stream, tr.pdl(), keys, rank, npad, sorted);
         tr.mark();
-        k_sp_heads<<<T, kSortThreads, 0, a.stream>>>(sorted, a.N, a.V, tilecnt);
+        launch_k(k_sp_heads, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V, tilecnt);
         tr.mark();
-        k_sp_segments<<<T, kSortThreads, 0, a.stream>>>(sorted, a.N, a.V, tilecnt, uniq, segoff, perm,
-                                                        segidx, slot, sc);
+        launch_k(k_sp_segments, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V,
+                 tilecnt, uniq, segoff, perm, segidx, slot, sc);
         tr.mark();
     } else {
         // no ids: zero distinct ids and zero valid occurrences
         cudaMemsetAsync(&sc->n_unique, 0, 2 * sizeof(int32_t), a.stream);
+        tr.launched = false;  // the next kernel follows the memset in plain stream order
     }
 }
 
@@ -616,6 +757,7 @@ __global__ void k_sp_export(const int32_t *__restrict__ uniq, const int32_t *__r
                             const DevScalars *__restrict__ sc, int64_t N, int32_t *__restrict__ uniq_out,
                             int32_t *__restrict__ counts_out, int32_t *__restrict__ n_unique_out)
 {
+    grid_dep_wait();
     const int U = sc->n_unique;
     for (int64_t u = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; u < N;
          u += (int64_t)gridDim.x * blockDim.x) {
@@ -642,6 +784,7 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     auto *slot = reinterpret_cast<int32_t *>(ws + L.sp_slot);
     auto *rowpart = reinterpret_cast<float *>(ws + L.sp_rowpart);
     auto *carry = reinterpret_cast<float *>(ws + L.sp_carry);
+    auto *bounds = reinterpret_cast<int32_t *>(ws + L.sp_bounds);
     auto *S = reinterpret_cast<float *>(ws + L.sp_rows);
     auto *colpart = reinterpret_cast<float *>(ws + L.colpart);
     auto *rsum_part = reinterpret_cast<double *>(ws + L.rsum_part);
@@ -654,27 +797,28 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     tr.mark();
     launch_sort_dedup(a, tr);
     const int G = kGridCtas;
-    k_sp_chunks<VEC><<<G, kThreads, 0, a.stream>>>(a.rows, perm, segidx, segoff, sc, S, rowpart, carry,
-                                                   colpart, D, NS);
+    const int nw = G / NS;
+    launch_k(k_sp_segsum<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), a.rows, perm, segidx, sc, S,
+             rowpart, carry, colpart, bounds, D, NS);
     tr.mark();
-    k_sp_carry<VEC><<<G, kThreads, 0, a.stream>>>(segoff, sc, carry, S, rowpart, colpart + (int64_t)G * D,
-                                                  D, NS);
+    launch_k(k_sp_carry<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), segidx, segoff, bounds, sc,
+             carry, S, rowpart, colpart + (int64_t)G * D, D, NS, nw);
     tr.mark();
     const int64_t vb = (a.V + kThreads - 1) / kThreads;
     const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
-    k_sp_vpass<<<GV, kThreads, 0, a.stream>>>(a.r, slot, rowpart, NS, a.V, D, a.beta2, a.one_minus_beta2,
-                                              rsum_part);
+    launch_k(k_sp_vpass, dim3(GV), dim3(kThreads), 0, a.stream, tr.pdl(), a.r, slot, rowpart, NS, a.V, D,
+             a.beta2, a.one_minus_beta2, rsum_part);
     tr.mark();
     launch_state(colpart, 2 * G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
-                 a.inv_bc, a.stream);
+                 a.inv_bc, a.stream, tr.pdl());
     tr.mark();
     const size_t cs_bytes = (size_t)D * sizeof(float);
     if (a.wbf16)
-        k_sp_apply<VEC, CPT, R, true><<<G, kThreads, cs_bytes, a.stream>>>(
-            a.W, S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+        launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(G), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
+                 S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
     else
-        k_sp_apply<VEC, CPT, R, false><<<G, kThreads, cs_bytes, a.stream>>>(
-            a.W, S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+        launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(G), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
+                 S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
     tr.mark();
     return cudaGetLastError();
 }
@@ -714,8 +858,8 @@ cudaError_t launch_sparse_unique(const SparseArgs &a, int32_t *uniq_out, int32_t
         nb = 1;
     if (nb > 4 * kGridCtas)
         nb = 4 * kGridCtas;
-    k_sp_export<<<(int)nb, kThreads, 0, a.stream>>>(uniq, segoff, sc, a.N, uniq_out, counts_out,
-                                                     n_unique_out);
+    launch_k(k_sp_export, dim3((int)nb), dim3(kThreads), 0, a.stream, tr.pdl(), uniq, segoff, sc, a.N,
+             uniq_out, counts_out, n_unique_out);
     // the touched-row map must be all-zero again before the next step
     int32_t *slot = reinterpret_cast<int32_t *>(a.ws + a.lay.sp_slot);
     cudaMemsetAsync(slot, 0, sizeof(int32_t) * (size_t)a.V, a.stream);
