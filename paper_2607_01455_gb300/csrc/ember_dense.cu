@@ -197,60 +197,106 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     }
 }
 
-// Pass 2: column EMA and the normaliser.  CTA x owns columns
-// [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in order.
+// Pass 2: column EMA and the normaliser.  The first nstate CTAs each own
+// columns [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in
+// order.  For the sparse step the remaining CTAs also do the row pass: r for
+// every row (rows outside the batch see a zero gradient row, touched rows
+// take their sum of g^2 per column slice from `rowpart`) and the sum of the
+// new r per CTA.  The last CTA to finish forms mean(rhat), mean(chat) and s.
+struct RowPass {
+    float *r;               // r[V], updated (sparse step only)
+    int32_t *slot;          // touched-row map, cleared here
+    const float *rowpart;   // per (distinct id, slice) sums of g^2
+    int nslices;
+    int nrow_ctas;          // 0 for the dense step
+};
+
 __global__ void __launch_bounds__(kStateThreads)
-k_state_dense(const float *__restrict__ colpart, int nparts, const double *__restrict__ rsum_part,
+k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict__ rsum_part,
               int nrsum, float *__restrict__ c, double *__restrict__ csum_part, DevScalars *sc,
-              int64_t V, int D, double beta2, double one_minus_beta2, double inv_bc)
+              int64_t V, int D, double beta2, double one_minus_beta2, double inv_bc, RowPass rowp)
 {
     constexpr int kW = kStateThreads / 32;
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
-    const int j = blockIdx.x * kStateCols + lane;
+    const int nstate = (int)gridDim.x - rowp.nrow_ctas;
     __shared__ double part[kW][32];
     __shared__ bool am_last;
-    grid_dep_wait();  // column partials and row sums of the reduce pass
+    grid_dep_wait();  // column partials and row sums of the earlier passes
     grid_dep_launch();
 
-    // rows w, w + 8, w + 16, ...: sixteen loads in flight, summed pairwise
-    // in fp32 within the batch and in fp64 across batches
-    constexpr int kBatch = 16;
-    double acc = 0.0;
-    if (j < D)
-        for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
-            float v[kBatch];
+    if ((int)blockIdx.x < nstate) {
+        const int j = blockIdx.x * kStateCols + lane;
+        // rows w, w + 8, w + 16, ...: sixteen loads in flight, summed pairwise
+        // in fp32 within the batch and in fp64 across batches
+        constexpr int kBatch = 16;
+        double acc = 0.0;
+        if (j < D)
+            for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
+                float v[kBatch];
 #pragma unroll
-            for (int k = 0; k < kBatch; ++k) {
-                const int b = b0 + k * kW;
-                v[k] = (b < nparts) ? __ldcg(colpart + (int64_t)b * D + j) : 0.f;
+                for (int k = 0; k < kBatch; ++k) {
+                    const int b = b0 + k * kW;
+                    v[k] = (b < nparts) ? __ldcg(colpart + (int64_t)b * D + j) : 0.f;
+                }
+#pragma unroll
+                for (int h = kBatch / 2; h >= 1; h >>= 1)
+#pragma unroll
+                    for (int k = 0; k < h; ++k)
+                        v[k] += v[k + h];
+                acc += (double)v[0];
+            }
+        part[w][lane] = acc;
+        __syncthreads();
+        if (w == 0) {
+            double tot = 0.0;
+#pragma unroll
+            for (int q = 0; q < kW; ++q)
+                tot += part[q][lane];
+            double cn = 0.0;
+            if (j < D) {
+                const double mean_col = tot / (double)V;
+                const float cnew = (float)(beta2 * (double)c[j] + one_minus_beta2 * mean_col);
+                c[j] = cnew;
+                cn = (double)cnew;
             }
 #pragma unroll
-            for (int h = kBatch / 2; h >= 1; h >>= 1)
-#pragma unroll
-                for (int k = 0; k < h; ++k)
-                    v[k] += v[k + h];
-            acc += (double)v[0];
+            for (int o = 16; o >= 1; o >>= 1)
+                cn += __shfl_xor_sync(0xffffffffu, cn, o);
+            if (lane == 0)
+                csum_part[blockIdx.x] = cn;
         }
-    part[w][lane] = acc;
-    __syncthreads();
-    if (w == 0) {
-        double tot = 0.0;
-#pragma unroll
-        for (int q = 0; q < kW; ++q)
-            tot += part[q][lane];
-        double cn = 0.0;
-        if (j < D) {
-            const double mean_col = tot / (double)V;
-            const float cnew = (float)(beta2 * (double)c[j] + one_minus_beta2 * mean_col);
-            c[j] = cnew;
-            cn = (double)cnew;
+    } else {
+        const int rb = (int)blockIdx.x - nstate;
+        double rsum = 0.0;
+        for (int64_t i = (int64_t)rb * kStateThreads + threadIdx.x; i < V;
+             i += (int64_t)rowp.nrow_ctas * kStateThreads) {
+            const int sl = rowp.slot[i];
+            double mean_row = 0.0;
+            if (sl) {
+                const int64_t u = sl - 1;
+                float tot = 0.f;
+                for (int k = 0; k < rowp.nslices; ++k)
+                    tot += rowp.rowpart[u * rowp.nslices + k];
+                mean_row = (double)tot / (double)D;
+                rowp.slot[i] = 0;
+            }
+            const float rn = (float)(beta2 * (double)rowp.r[i] + one_minus_beta2 * mean_row);
+            rowp.r[i] = rn;
+            rsum += (double)rn;
         }
 #pragma unroll
         for (int o = 16; o >= 1; o >>= 1)
-            cn += __shfl_xor_sync(0xffffffffu, cn, o);
+            rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
         if (lane == 0)
-            csum_part[blockIdx.x] = cn;
+            part[w][0] = rsum;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            double t = 0.0;
+            for (int q = 0; q < kW; ++q)
+                t += part[q][0];
+            rsum_part[rb] = t;
+        }
     }
     double csum = 0.0, rsum = 0.0;
     if (threadIdx.x == 0) {
@@ -262,7 +308,7 @@ k_state_dense(const float *__restrict__ colpart, int nparts, const double *__res
     if (am_last && w == 0) {
         __threadfence();
         // lane l sums entries l, l + 32, ... in order, then a fixed butterfly
-        for (int b = lane; b < (int)gridDim.x; b += 32)
+        for (int b = lane; b < nstate; b += 32)
             csum += __ldcg(csum_part + b);
         for (int b = lane; b < nrsum; b += 32)
             rsum += __ldcg(rsum_part + b);
@@ -401,7 +447,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     if (a.trace)
         cudaEventRecord(a.trace[1], a.stream);
     e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                     a.one_minus_beta2, a.inv_bc, a.stream, pdl);
+                     a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
     if (e != cudaSuccess)
         return e;
     if (a.trace)
@@ -424,13 +470,15 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 
 }  // namespace
 
-cudaError_t launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum,
-                         float *c, double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl)
+cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, int nrsum, float *c,
+                         double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl,
+                         float *r_rows, int32_t *slot, const float *rowpart, int nslices, int nrow_ctas)
 {
     const int nstate = (D + kStateCols - 1) / kStateCols;
-    return launch_k(k_state_dense, dim3(nstate), dim3(kStateThreads), 0, stream, pdl, colpart, nparts,
-                    rsum_part, nrsum, c, csum_part, sc, V, D, beta2, one_minus_beta2, inv_bc);
+    RowPass rp{r_rows, slot, rowpart, nslices, nrow_ctas};
+    return launch_k(k_state_dense, dim3(nstate + nrow_ctas), dim3(kStateThreads), 0, stream, pdl, colpart,
+                    nparts, rsum_part, nrsum, c, csum_part, sc, V, D, beta2, one_minus_beta2, inv_bc, rp);
 }
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)

@@ -102,9 +102,12 @@ struct DenseArgs {
 
 cudaError_t launch_dense_step(const DenseArgs &a);
 
-cudaError_t launch_state(const float *colpart, int nparts, const double *rsum_part, int nrsum,
-                         float *c, double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl);
+// Column EMA and normaliser; with nrow_ctas > 0 the same launch also runs the
+// sparse step's row pass (r for all V rows from the per-slice sums of g^2).
+cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, int nrsum, float *c,
+                         double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
+                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl,
+                         float *r_rows, int32_t *slot, const float *rowpart, int nslices, int nrow_ctas);
 
 struct SparseArgs {
     int64_t V, D, N;

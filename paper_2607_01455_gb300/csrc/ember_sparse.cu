@@ -29,9 +29,9 @@
 //             counts are (a Zipf head id can own thousands of occurrences);
 //             a run that crosses worker boundaries leaves one piece per
 //             worker, which k_sp_carry adds in worker order.
-//   rows      k_sp_vpass: r for all V rows, the sums of new r per CTA, and the
-//             touched-row map cleared for the next step.
-//   state     the dense step's column/normaliser pass.
+//   state     the dense step's column/normaliser pass, whose launch also runs
+//             the row pass: r for all V rows, the sums of new r per CTA, and
+//             the touched-row map cleared for the next step.
 //   apply     k_sp_apply: the update of the touched rows only.
 //
 // Every kernel after the first is launched with programmatic dependent
@@ -570,49 +570,12 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
             out[col * VEC + e] = colacc[e];
 }
 
-// Row second moment of all V rows: untouched rows see a zero gradient row.
-__global__ void __launch_bounds__(kThreads)
-k_sp_vpass(float *__restrict__ r, int32_t *__restrict__ slot, const float *__restrict__ rowpart,
-           int NS, int64_t V, int D, double beta2, double one_minus_beta2,
-           double *__restrict__ rsum_part)
-{
-    __shared__ double sh[kThreads / 32];
-    grid_dep_wait();  // per-run sums of g^2
-    grid_dep_launch();
-    double rsum = 0.0;
-    for (int64_t i = (int64_t)blockIdx.x * kThreads + threadIdx.x; i < V;
-         i += (int64_t)gridDim.x * kThreads) {
-        const int s = slot[i];
-        double mean_row = 0.0;
-        if (s) {
-            const int64_t u = s - 1;
-            float tot = 0.f;
-            for (int k = 0; k < NS; ++k)
-                tot += rowpart[u * NS + k];
-            mean_row = (double)tot / (double)D;
-            slot[i] = 0;
-        }
-        const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
-        r[i] = rn;
-        rsum += (double)rn;
-    }
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1)
-        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
-    if ((threadIdx.x & 31) == 0)
-        sh[threadIdx.x >> 5] = rsum;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double s = 0.0;
-        for (int k = 0; k < kThreads / 32; ++k)
-            s += sh[k];
-        rsum_part[blockIdx.x] = s;
-    }
-}
-
 // The update of the touched rows: W[uniq[u]] from the summed row S[u].
+// Three CTAs per SM (two for the widest rows): each CTA has only a few rows,
+// so more of them are kept in flight at once.
+constexpr int apply_ctas_per_sm(int cpt) { return cpt >= 8 ? 2 : 3; }
 template <int VEC, int CPT, int R, bool BF16>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+__global__ void __launch_bounds__(kThreads, apply_ctas_per_sm(CPT))
 k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__restrict__ uniq,
            const float *__restrict__ r, const float *__restrict__ c,
            const DevScalars *__restrict__ sc, int D, int tpr, float inv_bc, float eps,
@@ -773,7 +736,7 @@ __global__ void k_sp_export(const int32_t *__restrict__ uniq, const int32_t *__r
 template <int VEC, int CPT>
 cudaError_t launch_sparse_t(const SparseArgs &a)
 {
-    constexpr int R = (8 / CPT) < 1 ? 1 : (8 / CPT);
+    constexpr int R = (4 / CPT) < 1 ? 1 : (4 / CPT);
     unsigned char *ws = a.ws;
     const Layout &L = a.lay;
     DevScalars *sc = reinterpret_cast<DevScalars *>(ws + L.scalars);
@@ -804,20 +767,19 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     launch_k(k_sp_carry<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), segidx, segoff, bounds, sc,
              carry, S, rowpart, colpart + (int64_t)G * D, D, NS, nw);
     tr.mark();
+    // row pass (all V rows) and column pass in one launch
     const int64_t vb = (a.V + kThreads - 1) / kThreads;
     const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
-    launch_k(k_sp_vpass, dim3(GV), dim3(kThreads), 0, a.stream, tr.pdl(), a.r, slot, rowpart, NS, a.V, D,
-             a.beta2, a.one_minus_beta2, rsum_part);
-    tr.mark();
     launch_state(colpart, 2 * G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
-                 a.inv_bc, a.stream, tr.pdl());
+                 a.inv_bc, a.stream, tr.pdl(), a.r, slot, rowpart, NS, GV);
     tr.mark();
     const size_t cs_bytes = (size_t)D * sizeof(float);
+    const int GA = kSms * apply_ctas_per_sm(CPT);
     if (a.wbf16)
-        launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(G), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
+        launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
                  S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
     else
-        launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(G), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
+        launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
                  S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
     tr.mark();
     return cudaGetLastError();
