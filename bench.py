@@ -126,6 +126,33 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
             "kernels_ms": per, "ms_per_step_traced": ms_traced, "gpu_launches": nk * steps}
 
 
+def run_row_only(wl, dev, steps, warmup, flush, W, G):
+    """The row-only variant (vtil = rhat, one fused pass over G and W) on the
+    same table: 4VD + 2wVD + 8(V + D) algorithmic bytes per step."""
+    import torch
+    from paper_2607_01455_gb300.ember import Ember
+    emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, variant="row", device=dev)
+    t = 0
+    for _ in range(warmup):
+        t += 1
+        flush.zero_()
+        emb.step_dense(W, G, wl.lr, t)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for k in range(steps):
+        t += 1
+        flush.zero_()
+        ev[k][0].record()
+        emb.step_dense(W, G, wl.lr, t)
+        ev[k][1].record()
+    torch.cuda.synchronize()
+    if emb.device_status() != 0:
+        raise SystemExit("device status after the row-only steps")
+    ms = sum(a.elapsed_time(b) for a, b in ev) / steps
+    B = (4 + 2 * wbytes(wl)) * wl.V * wl.D + 8 * (wl.V + wl.D)
+    return {"variant": "row", "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
+            "algorithmic_bytes": B, "params_per_s": wl.V * wl.D / (ms * 1e-3), "gpu_launches": 2 * steps}
+
+
 def measured_hbm_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -412,6 +439,11 @@ def run_ours(args, world, rank, local):
                "sample": f"3 oracle dense steps on the first {rows} of {wl.V} rows (D={wl.D}), one thread",
                "ms_per_step": sec * 1e3}
 
+    row_only = None
+    if not args.no_row_only:
+        row_only = run_row_only(wl, dev, max(2 * TRACE_EVERY, min(args.steps, 100)), args.warmup, flush, W, G)
+        row_only["frac_of_measured_hbm"] = row_only["value"] / peak
+
     sparse = None
     if not args.no_sparse:
         swl = synth.WORKLOADS["sparse_v262144_d2048_bf16_n32768"]
@@ -440,6 +472,7 @@ def run_ours(args, world, rank, local):
         "timing": f"step time: CUDA events around each untraced step; kernel times: every {TRACE_EVERY}th step records events at kernel boundaries",
         "wall_s_timed_region": wall,
         "sparse": sparse,
+        "row_only": row_only,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -456,6 +489,7 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sparse", action="store_true")
+    ap.add_argument("--no-row-only", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -419,6 +419,160 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
     }
 }
 
+// Row-only Ember in one pass (variant ROW: vtil_ij = rhat_i, the "row-only"
+// row of the Section 2.1 ablation table).  The update of row i needs only
+// r_i, which depends on row i alone, so a CTA reads each row of G once,
+// finishes its sum of g^2 and its r_i, and updates the row of W from the
+// gradient still in registers: 4VD + 2wVD bytes instead of the full
+// preconditioner's 8VD + 2wVD.  Column sums of g^2 are still accumulated so
+// that c (part of the same V + D state) is maintained by the state pass.
+template <int VEC, int CPT, int R, bool BF16>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__restrict__ r,
+                float *__restrict__ colpart, double *__restrict__ rsum_part, int64_t V, int D, int tpr,
+                double beta2, double one_minus_beta2, float inv_bc, float eps, float lr_signed)
+{
+    using F = typename Vec<VEC>::F;
+    using WT = typename WRaw<BF16, VEC>::T;
+    constexpr int kWarps = kThreads / 32;
+    const int DV = D / VEC;
+    const int tid = threadIdx.x;
+    const int lane = tid & 31;
+    const int warp = tid >> 5;
+    const int rg = kThreads / tpr;
+    const int g = tid / tpr;
+    const int l = tid - g * tpr;
+    const int wpg = tpr >> 5;
+    const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
+    const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+    __shared__ float red[kWarps][R];
+    __shared__ float rs_sh[kThreads / 32 * R];  // sqrt(rhat) of this iteration's rows
+    __shared__ double rsum_sh[kWarps];
+    grid_dep_wait();
+    grid_dep_launch();
+
+    float acc[CPT][VEC];
+#pragma unroll
+    for (int c = 0; c < CPT; ++c)
+#pragma unroll
+        for (int e = 0; e < VEC; ++e)
+            acc[c][e] = 0.f;
+    double rsum = 0.0;
+    const int rows_per_it = rg * R;
+    for (int64_t base = row0; base < row1; base += rows_per_it) {
+        F v[R][CPT];
+        WT wr[R][CPT];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col = l + c * tpr;
+                const bool in = i < row1 && col < DV;
+                v[k][c] = in ? load_g<VEC>(G + i * D + (int64_t)col * VEC) : zero_vec<VEC>();
+                if (in)
+                    wr[k][c] = load_w<BF16, VEC>(W, i * D + (int64_t)col * VEC);
+            }
+        }
+        float rp[R];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            float s = 0.f;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c)
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const float x = comp(v[k][c], e);
+                    s = fmaf(x, x, s);
+                    acc[c][e] = fmaf(x, x, acc[c][e]);
+                }
+            rp[k] = s;
+        }
+        int row_in_warp;
+        const float tot = warp_sum_transposed<R>(rp, lane, row_in_warp);
+        if ((lane & (32 / R - 1)) == 0)
+            red[warp][row_in_warp] = tot;
+        __syncthreads();
+        if (l < R) {
+            const int64_t i = base + (int64_t)g * R + l;
+            float rsv = 0.f;
+            if (i < row1) {
+                float sum = 0.f;
+                for (int q = 0; q < wpg; ++q)
+                    sum += red[g * wpg + q][l];
+                const double mean_row = (double)sum / (double)D;
+                const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
+                r[i] = rn;
+                rsum += (double)rn;
+                rsv = sqrtf(rn * inv_bc);
+            }
+            rs_sh[g * R + l] = rsv;
+        }
+        __syncthreads();
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+            if (i >= row1)
+                continue;
+            const float den = rs_sh[g * R + k] + eps;
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col = l + c * tpr;
+                if (col >= DV)
+                    continue;
+                float w[VEC];
+                unpack_w(wr[k][c], w);
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    w[e] = fmaf(lr_signed, comp(v[k][c], e) / den, w[e]);
+                store_w<BF16, VEC>(W, i * D + (int64_t)col * VEC, w);
+            }
+        }
+    }
+
+    // column partial of this CTA: row groups combined in order 0 .. rg-1
+    float *out = colpart + (int64_t)blockIdx.x * D;
+    if (rg == 1) {
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+            const int col = l + c * tpr;
+            if (col < DV)
+#pragma unroll
+                for (int e = 0; e < VEC; ++e)
+                    out[col * VEC + e] = acc[c][e];
+        }
+    } else {
+        extern __shared__ float colsh[];  // D floats
+        for (int q = 0; q < rg; ++q) {
+            if (g == q) {
+#pragma unroll
+                for (int c = 0; c < CPT; ++c) {
+                    const int col = l + c * tpr;
+                    if (col < DV)
+#pragma unroll
+                        for (int e = 0; e < VEC; ++e)
+                            colsh[col * VEC + e] = (q == 0) ? acc[c][e] : colsh[col * VEC + e] + acc[c][e];
+                }
+            }
+            __syncthreads();
+        }
+        for (int j = tid; j < D; j += kThreads)
+            out[j] = colsh[j];
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+    if (lane == 0)
+        rsum_sh[warp] = rsum;
+    __syncthreads();
+    if (tid == 0) {
+        double t = 0.0;
+        for (int q = 0; q < kWarps; ++q)
+            t += rsum_sh[q];
+        rsum_part[blockIdx.x] = t;
+    }
+}
+
 template <int VEC, int CPT>
 cudaError_t launch_dense_t(const DenseArgs &a)
 {
@@ -438,6 +592,33 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     // dependent launch.
     const bool pdl = (a.trace == nullptr);
     cudaError_t e;
+    if (a.variant == EMBER_VARIANT_ROW) {
+        // one pass over G and W, then the column state; no apply pass
+        constexpr int RR = (4 / CPT) < 1 ? 1 : (4 / CPT);
+        if (a.trace)
+            cudaEventRecord(a.trace[0], a.stream);
+        if (a.wbf16)
+            e = launch_k(k_rowonly_dense<VEC, CPT, RR, true>, dim3(nparts), dim3(kThreads), shmem, a.stream,
+                         false, a.W, a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2,
+                         a.one_minus_beta2, (float)a.inv_bc, a.eps, a.lr_signed);
+        else
+            e = launch_k(k_rowonly_dense<VEC, CPT, RR, false>, dim3(nparts), dim3(kThreads), shmem, a.stream,
+                         false, a.W, a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2,
+                         a.one_minus_beta2, (float)a.inv_bc, a.eps, a.lr_signed);
+        if (e != cudaSuccess)
+            return e;
+        if (a.trace)
+            cudaEventRecord(a.trace[1], a.stream);
+        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        if (e != cudaSuccess)
+            return e;
+        if (a.trace) {
+            cudaEventRecord(a.trace[2], a.stream);
+            cudaEventRecord(a.trace[3], a.stream);
+        }
+        return cudaGetLastError();
+    }
     if (a.trace)
         cudaEventRecord(a.trace[0], a.stream);
     e = launch_k(k_reduce_dense<VEC, CPT, R1>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,

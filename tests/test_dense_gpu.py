@@ -72,6 +72,20 @@ def test_dense_parity_hyperparameters(cuda_device, opt, V, D):
         gated_dense_step(emb, W, rand_grad(V, D, t, cuda_device, seed=3), 2e-3, t, opt)
 
 
+@pytest.mark.parametrize("V,D,wdtype", [(305, 8192, "bf16"), (1000, 4096, "bf16"), (2049, 896, "bf16"),
+                                         (777, 203, "f32"), (3001, 64, "bf16"), (1, 8, "bf16"),
+                                         (7, 5, "f32")])
+def test_row_only_single_pass_parity(cuda_device, V, D, wdtype):
+    """The row-only variant runs as one fused pass over G and W; it must
+    still match the oracle's row-only step, state included."""
+    opt = Opt(variant="row")
+    emb = make(V, D, wdtype, opt)
+    W = rand_w(V, D, wdtype, cuda_device, seed=D)
+    for t in range(1, 4):
+        G = rand_grad(V, D, t, cuda_device, seed=V, zero_rows=[0] if V > 2 else [])
+        gated_dense_step(emb, W, G, 1e-3, t, opt)
+
+
 def test_dense_workload_small_all_steps(cuda_device):
     """The 1024 x 64 fp32 workload, all 10 steps, each gated."""
     wl = synth.WORKLOADS["dense_v1024_d64_f32"]
