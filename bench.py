@@ -211,29 +211,38 @@ class ClockSampler:
                 "samples": len(rows), "power_w_max": max(float(p[3]) for p in rows)}
 
 
-def oracle_sample(wl, rows, seed=0):
+class OracleSample:
     """The oracle's dense step on the first `rows` rows of the workload (a
-    rows x D table with the workload's generator); returns seconds."""
-    import numpy as np
-    import torch
-    import oracle
-    from paper_2607_01455_gb300 import synth
-    sub = synth.Workload(wl.name + "_sample", rows, wl.D, wl.wdtype, 1,
-                         zero_frac=wl.zero_frac, heavy_frac=wl.heavy_frac)
-    W = synth.init_weights(sub, seed, "cpu")
-    W = W.view(torch.int16).numpy().view(np.uint16).copy() if wl.wdtype == "bf16" else W.numpy().copy()
-    G = synth.dense_grad(sub, seed, 1, "cpu").numpy()
-    r = np.zeros(rows, np.float32)
-    c = np.zeros(wl.D, np.float32)
-    t0 = time.perf_counter()
-    oracle.step_dense(W, G, r, c, wl.lr, 1)
-    return time.perf_counter() - t0
+    rows x D table drawn with the workload's generator), stepped repeatedly."""
+
+    def __init__(self, wl, rows, seed=0):
+        import numpy as np
+        import torch
+        from paper_2607_01455_gb300 import synth
+        sub = synth.Workload(wl.name + "_sample", rows, wl.D, wl.wdtype, 1,
+                             zero_frac=wl.zero_frac, heavy_frac=wl.heavy_frac)
+        W = synth.init_weights(sub, seed, "cpu")
+        self.W = (W.view(torch.int16).numpy().view(np.uint16).copy() if wl.wdtype == "bf16"
+                  else W.numpy().copy())
+        self.G = synth.dense_grad(sub, seed, 1, "cpu").numpy()
+        self.r = np.zeros(rows, np.float32)
+        self.c = np.zeros(wl.D, np.float32)
+        self.lr, self.t, self.rows = wl.lr, 0, rows
+        self.bytes = step_bytes(sub)
+
+    def step(self):
+        """One oracle step; returns its seconds."""
+        import oracle
+        self.t += 1
+        t0 = time.perf_counter()
+        oracle.step_dense(self.W, self.G, self.r, self.c, self.lr, self.t)
+        return time.perf_counter() - t0
 
 
 def sample_rows_for(wl, seconds):
     """Rows of a sample whose oracle step takes about `seconds`."""
     probe = 64
-    dt = oracle_sample(wl, probe)
+    dt = OracleSample(wl, probe).step()
     return int(max(16, min(wl.V, probe * seconds / max(dt, 1e-6))))
 
 
@@ -268,14 +277,14 @@ def run_reference(args, world, rank):
     wl = synth.WORKLOADS[args.workload]
     if rank != 0:
         return 0
-    budget = 90.0  # seconds for the whole warm-up + timed run
+    budget = 90.0  # seconds of oracle work for the whole warm-up + timed run
     rows = sample_rows_for(wl, budget / (args.steps + args.warmup))
-    sub_bytes = step_bytes(synth.Workload("s", rows, wl.D, wl.wdtype, 1))
+    smp = OracleSample(wl, rows)
     for _ in range(args.warmup):
-        oracle_sample(wl, rows)
-    times = [oracle_sample(wl, rows) for _ in range(args.steps)]
+        smp.step()
+    times = [smp.step() for _ in range(args.steps)]
     sec = sum(times) / len(times)
-    gbs = sub_bytes / sec / 1e9
+    gbs = smp.bytes / sec / 1e9
     sample = f"oracle dense step on the first {rows} of {wl.V} rows (D={wl.D}, {wl.wdtype} W), one thread"
     line = {
         "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world,
@@ -405,12 +414,15 @@ def run_ours(args, world, rank, local):
         "algorithmic_bytes_per_launch": kb[dom],
     }
 
-    # end to end through the C ABI: pinned host gradient in, updated weights out
+    # end to end through the C ABI: the gradient comes in from pinned host
+    # memory, the step runs, and its result -- the optimizer state r, c
+    # (V + D floats) -- goes back to pinned host memory.  W stays on the
+    # device, as model weights do in training.
     e2e = None
     if not args.no_e2e:
-        n_e2e = max(1, min(args.steps, 5))
+        n_e2e = max(1, min(args.steps, 10))
         Gh = G.cpu().pin_memory()
-        Wh = torch.empty(W.shape, dtype=W.dtype, pin_memory=True)
+        Sh = torch.empty(emb.state.shape, dtype=emb.state.dtype, pin_memory=True)
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         G2 = torch.empty_like(G)
         ts = []
@@ -420,22 +432,23 @@ def run_ours(args, world, rank, local):
             e0.record(stream)
             G2.copy_(Gh, non_blocking=True)
             emb.step_dense(W, G2, wl.lr, t)
-            Wh.copy_(W, non_blocking=True)
+            Sh.copy_(emb.state, non_blocking=True)
             e1.record(stream)
             e1.synchronize()
             ts.append(e0.elapsed_time(e1))
         ms_e2e = allreduce_max(world, sum(ts) / len(ts))
         e2e = {"value": world * B / (ms_e2e * 1e-3) / 1e9, "unit": "GB/s",
-               "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": W.numel() * W.element_size(),
-               "ms_per_step": ms_e2e, "steps": n_e2e}
+               "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": emb.state.numel() * 4,
+               "ms_per_step": ms_e2e, "steps": n_e2e,
+               "what": "pinned-host G -> device, dense step through the C ABI, state r,c -> pinned host"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         rows = sample_rows_for(wl, 5.0)
-        secs = [oracle_sample(wl, rows) for _ in range(3)]
-        sub = synth.Workload("s", rows, wl.D, wl.wdtype, 1)
+        smp = OracleSample(wl, rows)
+        secs = [smp.step() for _ in range(3)]
         sec = sum(secs) / len(secs)
-        cpu = {"value": step_bytes(sub) / sec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+        cpu = {"value": smp.bytes / sec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"3 oracle dense steps on the first {rows} of {wl.V} rows (D={wl.D}), one thread",
                "ms_per_step": sec * 1e3}
 

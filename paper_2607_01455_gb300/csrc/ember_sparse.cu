@@ -50,57 +50,97 @@ using namespace dev;
 constexpr uint64_t kPad = ~0ull;
 constexpr int kKeysPerThread = kSortTile / kSortThreads;
 
+// keys a <= b afterwards when `up`, a >= b otherwise
+__device__ __forceinline__ void cmp_swap(uint64_t &a, uint64_t &b, bool up)
+{
+    if ((a > b) == up) {
+        const uint64_t x = a;
+        a = b;
+        b = x;
+    }
+}
+
+__device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t x, int m)
+{
+    const uint32_t lo = __shfl_xor_sync(0xffffffffu, (uint32_t)x, m);
+    const uint32_t hi = __shfl_xor_sync(0xffffffffu, (uint32_t)(x >> 32), m);
+    return ((uint64_t)hi << 32) | lo;
+}
+
+// Bitonic sort of one tile of kSortTile keys, thread t holding keys
+// 4t .. 4t + 3.  For the compare-exchange of keys i and i ^ j at merge size
+// k, both holders keep min or max by the same rule: the lower index of the
+// pair keeps the min when the block (i & k) sorts ascending.  Partners at
+// distance 1 or 2 are in the same thread, distance 4 .. 64 in the same warp
+// (shuffles), and only distances 128 .. 512 go through shared memory.
 template <typename IdT>
 __global__ void __launch_bounds__(kSortThreads)
 k_sp_tile_sort(const IdT *__restrict__ ids, int64_t N, int64_t V, uint64_t *__restrict__ keys,
                int32_t *__restrict__ rank, DevScalars *sc)
 {
+    static_assert(kSortTile == 4 * kSortThreads, "four keys per thread");
     __shared__ uint64_t s[kSortTile];
     const int64_t base = (int64_t)blockIdx.x * kSortTile;
-    bool bad = false;
+    const int t = threadIdx.x;
     grid_dep_wait();  // first kernel of a step: returns at once
     grid_dep_launch();
+    bool bad = false;
+    uint64_t key[4];
 #pragma unroll
-    for (int q = 0; q < kKeysPerThread; ++q) {
-        const int i = threadIdx.x + q * kSortThreads;
-        const int64_t k = base + i;
-        uint64_t key = kPad;
+    for (int q = 0; q < 4; ++q) {
+        const int64_t k = base + 4 * t + q;
+        key[q] = kPad;
         if (k < N) {
             int64_t id = (int64_t)ids[k];
             if (id < 0 || id >= V) {  // skipped: sorts after every valid id
                 bad = true;
                 id = V;
             }
-            key = ((uint64_t)id << 32) | (uint64_t)k;
+            key[q] = ((uint64_t)id << 32) | (uint64_t)k;
         }
-        s[i] = key;
     }
     if (bad)
         atomicOr(&sc->flags, kFlagIdRange);
-    __syncthreads();
-    for (int lk = 1; (1 << lk) <= kSortTile; ++lk) {
-        for (int lj = lk - 1; lj >= 0; --lj) {
-            const int j = 1 << lj;
+
+    for (int k = 2; k <= kSortTile; k <<= 1) {
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            if (j >= 128) {  // partner in another warp
 #pragma unroll
-            for (int q = 0; q < kSortTile / 2 / kSortThreads; ++q) {
-                const int p = threadIdx.x + q * kSortThreads;  // pair index
-                const int i = ((p >> lj) << (lj + 1)) | (p & (j - 1));
-                const int l = i + j;
-                const bool up = ((i >> lk) & 1) == 0;
-                const uint64_t a = s[i], b = s[l];
-                if ((a > b) == up) {
-                    s[i] = b;
-                    s[l] = a;
+                for (int q = 0; q < 4; ++q)
+                    s[4 * t + q] = key[q];
+                __syncthreads();
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int i = 4 * t + q;
+                    const uint64_t o = s[i ^ j];
+                    const bool keep_min = ((i & j) == 0) == ((i & k) == 0);
+                    key[q] = keep_min ? (key[q] < o ? key[q] : o) : (key[q] > o ? key[q] : o);
+                }
+                __syncthreads();
+            } else if (j >= 4) {  // partner in this warp
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const int i = 4 * t + q;
+                    const uint64_t o = shfl_xor_u64(key[q], j >> 2);
+                    const bool keep_min = ((i & j) == 0) == ((i & k) == 0);
+                    key[q] = keep_min ? (key[q] < o ? key[q] : o) : (key[q] > o ? key[q] : o);
+                }
+            } else {  // partner in this thread: pairs (0,1),(2,3) or (0,2),(1,3)
+                const bool up = ((4 * t) & k) == 0;  // for k >= 4 the same for all four keys
+                if (j == 1) {
+                    cmp_swap(key[0], key[1], k == 2 ? (((4 * t) & 2) == 0) : up);
+                    cmp_swap(key[2], key[3], k == 2 ? (((4 * t + 2) & 2) == 0) : up);
+                } else {
+                    cmp_swap(key[0], key[2], up);
+                    cmp_swap(key[1], key[3], up);
                 }
             }
-            __syncthreads();
         }
     }
 #pragma unroll
-    for (int q = 0; q < kKeysPerThread; ++q) {
-        const int i = threadIdx.x + q * kSortThreads;
-        keys[base + i] = s[i];
-        rank[base + i] = i;
+    for (int q = 0; q < 4; ++q) {
+        keys[base + 4 * t + q] = key[q];
+        rank[base + 4 * t + q] = 4 * t + q;
     }
 }
 
