@@ -32,9 +32,10 @@ FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
 
 # dram__bytes_read.sum + dram__bytes_write.sum per launch of the apply kernel
-# on the default workload, from the ncu capture summarised in profiles/
-# (None until a capture of the current kernel exists).
-APPLY_TRAFFIC_BYTES = None
+# on the default workload (V=128256, D=8192, bf16 W), from the one-pass ncu
+# capture summarised in profiles/dense_lmhead_v128256_d8192_bf16_launches.md.
+# Set to None whenever k_apply_dense changes until it is captured again.
+APPLY_TRAFFIC_BYTES = 8374871296
 
 
 def wbytes(wl):

@@ -214,3 +214,28 @@ def test_sparse_workload_262144x2048(cuda_device):
         else:
             emb.step_sparse(W, ids, rows, wl.lr, t)
     assert emb.device_status() == 0
+
+
+def test_sparse_graph_capture_matches_eager(cuda_device):
+    """A sparse step is a fixed sequence of launches for a given N, so it can be
+    captured in a CUDA graph; replaying it gives the eager result bit for bit."""
+    V, D, N = 20000, 512, 9000
+    e1, e2 = make(V, D, "bf16", N), make(V, D, "bf16", N)
+    W0 = (torch.randn(V, D, device=cuda_device) * 0.02).to(torch.bfloat16)
+    W1, W2 = W0.clone(), W0.clone()
+    ids, rows = batch(V, D, N, 1, cuda_device, seed=4)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        e2.step_sparse(W2, ids, rows, 1e-3, 1, stream=s)  # warm-up outside the capture
+    torch.cuda.synchronize()
+    W2.copy_(W0)
+    e2.state.zero_()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        e2.step_sparse(W2, ids, rows, 1e-3, 1, stream=s)
+    graph.replay()
+    e1.step_sparse(W1, ids, rows, 1e-3, 1)
+    torch.cuda.synchronize()
+    assert torch.equal(W1.view(torch.int16), W2.view(torch.int16))
+    assert torch.equal(e1.state, e2.state)
