@@ -26,7 +26,7 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
     L.scalars = take(sizeof(DevScalars));
     L.rsum_part = take(sizeof(double) * kGridCtas);
     L.csum_part = take(sizeof(double) * nstate);
-    L.colpart = take(sizeof(float) * 2 * (size_t)kGridCtas * (size_t)D);
+    L.colpart = take(sizeof(float) * (size_t)kPartRows * (size_t)D);
     if (max_sparse_N > 0) {
         const size_t N = (size_t)max_sparse_N;
         const size_t Npad = (N + kSortTile - 1) / kSortTile * kSortTile;
@@ -40,9 +40,10 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
         L.sp_uniq = take(sizeof(int32_t) * N);
         L.sp_segoff = take(sizeof(int32_t) * (N + 1));
         L.sp_slot = take(sizeof(int32_t) * (size_t)V);
+        L.sp_single = take(sizeof(int32_t) * N);
         L.sp_rowpart = take(sizeof(float) * N * nslices);
-        L.sp_carry = take(sizeof(float) * 2 * (size_t)kGridCtas * (size_t)D);
-        L.sp_bounds = take(sizeof(int32_t) * ((size_t)kGridCtas + 1));
+        L.sp_carry = take(sizeof(float) * 2 * (size_t)kSparseCtas * (size_t)D);
+        L.sp_bounds = take(sizeof(int32_t) * ((size_t)kSparseCtas + 1));
         L.sp_rows = take(sizeof(float) * N * (size_t)D);
     }
     L.total = off;

@@ -19,6 +19,10 @@ constexpr int kThreads = 256;
 constexpr int kCtasPerSm = 2;
 constexpr int kSms = 152;
 constexpr int kGridCtas = kSms * kCtasPerSm;
+// The sparse step's segment sums run three smaller CTAs per SM.
+constexpr int kSparseCtasPerSm = 3;
+constexpr int kSparseCtas = kSms * kSparseCtasPerSm;
+constexpr int kPartRows = kSparseCtas > kGridCtas ? kSparseCtas : kGridCtas;
 
 // The state pass reduces 32 columns per CTA.
 constexpr int kStateCols = 32;
@@ -51,7 +55,7 @@ struct Layout {
     size_t scalars;     // DevScalars
     size_t rsum_part;   // double[kGridCtas]            sum of new r per CTA
     size_t csum_part;   // double[ceil(D/32)]           sum of new c per state CTA
-    size_t colpart;     // float[2 * kGridCtas * D]     column sums of g^2 per CTA
+    size_t colpart;     // float[kPartRows * D]     column sums of g^2 per CTA
     // sparse step (present when max_sparse_N > 0); N = max_sparse_N,
     // Npad = N rounded up to kSortTile
     size_t sp_keys;     // uint64[Npad]  (id << 32 | occurrence), sorted within tiles
@@ -63,10 +67,11 @@ struct Layout {
     size_t sp_uniq;     // int32[N]      distinct ids, ascending
     size_t sp_segoff;   // int32[N + 1]  first sorted position of each distinct id
     size_t sp_slot;     // int32[V]      1 + distinct-id index of a touched row, else 0
+    size_t sp_single;   // int32[N]      occurrence index of an id seen once, else -1
     size_t sp_rowpart;  // float[N * ceil(D / kThreads)]  sum g^2 per (distinct id, slice)
-    size_t sp_carry;    // float[2 * kGridCtas * D]  partial sums of runs cut by worker ranges
-    size_t sp_bounds;   // int32[kGridCtas + 1]  first sorted position of each worker range
-    size_t sp_rows;     // float[N * D]  summed gradient row of each distinct id
+    size_t sp_carry;    // float[2 * kSparseCtas * D]  partial sums of runs cut by worker ranges
+    size_t sp_bounds;   // int32[kSparseCtas + 1]  first sorted position of each worker range
+    size_t sp_rows;     // float[N * D]  summed gradient row of each distinct id seen twice or more
     size_t total;
 };
 

@@ -243,7 +243,7 @@ __global__ void __launch_bounds__(kSortThreads)
 k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
               const int32_t *__restrict__ tilecnt, int32_t *__restrict__ uniq,
               int32_t *__restrict__ segoff, int32_t *__restrict__ perm, int32_t *__restrict__ segidx,
-              int32_t *__restrict__ slot, DevScalars *sc)
+              int32_t *__restrict__ slot, int32_t *__restrict__ single, DevScalars *sc)
 {
     __shared__ int pre[2];
     __shared__ int wsum[kSortThreads / 32];
@@ -301,6 +301,9 @@ k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
             uniq[run] = id;
             segoff[run] = (int)p;
             slot[id] = run + 1;
+            // an id seen once: its summed row is that occurrence's row
+            const bool once = p + 1 >= N || (sorted[p + 1] >> 32) != (uint64_t)id;
+            single[run] = once ? (int)(key[q] & 0xffffffffu) : -1;
             ++run;
         }
         if (valid[q]) {
@@ -381,14 +384,14 @@ __device__ __forceinline__ int worker_of(int p, int u, int nw, int64_t C)
 // first run, slot 1: its last run); k_sp_carry adds the pieces in worker
 // order.  Completed runs are written to S with their sum of g^2 per slice.
 template <int VEC>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+__global__ void __launch_bounds__(kThreads, kSparseCtasPerSm)
 k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             const int32_t *__restrict__ segidx, const DevScalars *__restrict__ sc,
             float *__restrict__ S, float *__restrict__ rowpart, float *__restrict__ carry,
             float *__restrict__ colpart, int32_t *__restrict__ bounds, int D, int NS)
 {
     using F = typename Vec<VEC>::F;
-    constexpr int R = 16;
+    constexpr int R = 8;  // rows in flight per thread
     constexpr int kWarps = kThreads / 32;
     constexpr int kFin = 32;  // completed runs buffered before their g^2 sums are written
     __shared__ float rp[kFin][kWarps];
@@ -446,6 +449,7 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
         const bool first_cut = p0 > 0 && segidx[p0 - 1] == u_first;
         const bool last_cut = p1 < n_valid && segidx[p1] == u_last;
         int cur = u_first;
+        int len = 0;  // occurrences of `cur` seen in this range
         F acc = zero_vec<VEC>();
         auto flush = [&](int u) {
             const bool before = first_cut && u == u_first;
@@ -453,7 +457,9 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             if (!before && !after) {
                 float ps = 0.f;
                 if (active) {
-                    *reinterpret_cast<F *>(S + (int64_t)u * D + (int64_t)col * VEC) = acc;
+                    // an id seen once needs no summed row: the apply reads its occurrence row
+                    if (len > 1)
+                        *reinterpret_cast<F *>(S + (int64_t)u * D + (int64_t)col * VEC) = acc;
 #pragma unroll
                     for (int e = 0; e < VEC; ++e) {
                         const float a = comp(acc, e);
@@ -498,7 +504,9 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                     flush(cur);
                     acc = zero_vec<VEC>();
                     cur = uu[k];
+                    len = 0;
                 }
+                ++len;
 #pragma unroll
                 for (int e = 0; e < VEC; ++e)
                     set_comp(acc, e, comp(acc, e) + comp(v[k], e));
@@ -524,7 +532,7 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
 // pieces -- the previous worker's last piece, then the first pieces of the
 // following workers up to the one holding the run's end -- in worker order.
 template <int VEC>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+__global__ void __launch_bounds__(kThreads, kSparseCtasPerSm)
 k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segoff,
            const int32_t *__restrict__ bounds, const DevScalars *__restrict__ sc,
            const float *__restrict__ carry, float *__restrict__ S, float *__restrict__ rowpart,
@@ -600,14 +608,15 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
             rowpart[(int64_t)u * NS + sigma] = t;
         }
     }
-    float *out = colpart + (int64_t)blockIdx.x * D;
-    for (int j = threadIdx.x; j < D; j += kThreads)
-        out[j] = 0.f;
-    __syncthreads();
-    if (active && mine)
+    // CTA b of this kernel and CTA b of k_sp_segsum share worker bd - 1 and
+    // slice sigma: add this run's column sums to that CTA's partial row
+    // (its value plus this one, in that order)
+    if (active && mine) {
+        float *out = colpart + (int64_t)blockIdx.x * D;
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
-            out[col * VEC + e] = colacc[e];
+            out[col * VEC + e] += colacc[e];
+    }
 }
 
 // The update of the touched rows: W[uniq[u]] from the summed row S[u].
@@ -616,7 +625,8 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
 constexpr int apply_ctas_per_sm(int cpt) { return cpt >= 8 ? 2 : 3; }
 template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, apply_ctas_per_sm(CPT))
-k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__restrict__ uniq,
+k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__restrict__ rows,
+           const int32_t *__restrict__ uniq, const int32_t *__restrict__ single,
            const float *__restrict__ r, const float *__restrict__ c,
            const DevScalars *__restrict__ sc, int D, int tpr, float inv_bc, float eps,
            float lr_signed, int variant)
@@ -639,11 +649,15 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__r
 
     const int64_t stride = (int64_t)gridDim.x * rg * R;
     const int64_t ub0 = ((int64_t)blockIdx.x * rg + g) * R;
-    // row ids of the next iteration are loaded while this one's rows are in flight
+    // row ids (and, for ids seen once, the occurrence row) of the next
+    // iteration are loaded while this one's rows are in flight
     int64_t next[R];
+    int nsingle[R];
 #pragma unroll
-    for (int k = 0; k < R; ++k)
+    for (int k = 0; k < R; ++k) {
         next[k] = (ub0 + k < U) ? (int64_t)uniq[ub0 + k] : -1;
+        nsingle[k] = (ub0 + k < U) ? single[ub0 + k] : -1;
+    }
     for (int64_t ub = ub0; ub < U; ub += stride) {
         F gv[R][CPT];
         WT wr[R][CPT];
@@ -652,11 +666,12 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__r
         for (int k = 0; k < R; ++k) {
             const int64_t u = ub + k;
             row[k] = next[k];
+            const float *src = (nsingle[k] >= 0) ? rows + (int64_t)nsingle[k] * D : S + u * D;
 #pragma unroll
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (row[k] >= 0 && col < DV) {
-                    gv[k][cc] = load_g<VEC>(S + u * D + (int64_t)col * VEC);
+                    gv[k][cc] = load_g<VEC>(src + (int64_t)col * VEC);
                     wr[k][cc] = load_w<BF16, VEC>(W, row[k] * D + (int64_t)col * VEC);
                 }
             }
@@ -665,6 +680,7 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const int32_t *__r
         for (int k = 0; k < R; ++k) {
             const int64_t un = ub + stride + k;
             next[k] = (un < U) ? (int64_t)uniq[un] : -1;
+            nsingle[k] = (un < U) ? single[un] : -1;
         }
 #pragma unroll
         for (int k = 0; k < R; ++k) {
@@ -726,6 +742,7 @@ void launch_sort_dedup(const SparseArgs &a, Tracer &tr)
     auto *uniq = reinterpret_cast<int32_t *>(ws + L.sp_uniq);
     auto *segoff = reinterpret_cast<int32_t *>(ws + L.sp_segoff);
     auto *slot = reinterpret_cast<int32_t *>(ws + L.sp_slot);
+    auto *single = reinterpret_cast<int32_t *>(ws + L.sp_single);
     if (a.N > 0) {
         const int T = (int)((a.N + kSortTile - 1) / kSortTile);
         const int64_t npad = (int64_t)T * kSortTile;
@@ -746,7 +763,7 @@ void launch_sort_dedup(const SparseArgs &a, Tracer &tr)
         launch_k(k_sp_heads, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V, tilecnt);
         tr.mark();
         launch_k(k_sp_segments, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V,
-                 tilecnt, uniq, segoff, perm, segidx, slot, sc);
+                 tilecnt, uniq, segoff, perm, segidx, slot, single, sc);
         tr.mark();
     } else {
         // no ids: zero distinct ids and zero valid occurrences
@@ -785,6 +802,7 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     auto *uniq = reinterpret_cast<int32_t *>(ws + L.sp_uniq);
     auto *segoff = reinterpret_cast<int32_t *>(ws + L.sp_segoff);
     auto *slot = reinterpret_cast<int32_t *>(ws + L.sp_slot);
+    auto *single = reinterpret_cast<int32_t *>(ws + L.sp_single);
     auto *rowpart = reinterpret_cast<float *>(ws + L.sp_rowpart);
     auto *carry = reinterpret_cast<float *>(ws + L.sp_carry);
     auto *bounds = reinterpret_cast<int32_t *>(ws + L.sp_bounds);
@@ -799,28 +817,30 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
 
     tr.mark();
     launch_sort_dedup(a, tr);
-    const int G = kGridCtas;
+    const int G = kSparseCtas;
     const int nw = G / NS;
     launch_k(k_sp_segsum<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), a.rows, perm, segidx, sc, S,
              rowpart, carry, colpart, bounds, D, NS);
     tr.mark();
     launch_k(k_sp_carry<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), segidx, segoff, bounds, sc,
-             carry, S, rowpart, colpart + (int64_t)G * D, D, NS, nw);
+             carry, S, rowpart, colpart, D, NS, nw);
     tr.mark();
     // row pass (all V rows) and column pass in one launch
     const int64_t vb = (a.V + kThreads - 1) / kThreads;
     const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
-    launch_state(colpart, 2 * G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
+    launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
                  a.inv_bc, a.stream, tr.pdl(), a.r, slot, rowpart, NS, GV);
     tr.mark();
     const size_t cs_bytes = (size_t)D * sizeof(float);
     const int GA = kSms * apply_ctas_per_sm(CPT);
     if (a.wbf16)
         launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
-                 S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+                 S, a.rows, uniq, single, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                 a.variant);
     else
         launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
-                 S, uniq, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed, a.variant);
+                 S, a.rows, uniq, single, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                 a.variant);
     tr.mark();
     return cudaGetLastError();
 }
