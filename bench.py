@@ -437,11 +437,27 @@ def run_ours(args, world, rank, local):
             e1.record(stream)
             e1.synchronize()
             ts.append(e0.elapsed_time(e1))
+        ms_copy = allreduce_max(world, sum(ts) / len(ts))
+        # the same, with the reduce pass reading G over the chip-to-chip link
+        # and staging it in HBM (ember_step_dense_from_host): no copy engine
+        ts = []
+        for _ in range(n_e2e):
+            t += 1
+            flush.zero_()
+            e0.record(stream)
+            emb.step_dense_from_host(W, Gh, G2, wl.lr, t)
+            Sh.copy_(emb.state, non_blocking=True)
+            e1.record(stream)
+            e1.synchronize()
+            ts.append(e0.elapsed_time(e1))
         ms_e2e = allreduce_max(world, sum(ts) / len(ts))
         e2e = {"value": world * B / (ms_e2e * 1e-3) / 1e9, "unit": "GB/s",
                "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": emb.state.numel() * 4,
                "ms_per_step": ms_e2e, "steps": n_e2e,
-               "what": "pinned-host G -> device, dense step through the C ABI, state r,c -> pinned host"}
+               "what": "pinned-host G read by the reduce pass over the chip-to-chip link and staged in "
+                       "HBM (ember_step_dense_from_host), state r,c -> pinned host",
+               "copy_engine": {"ms_per_step": ms_copy, "value": world * B / (ms_copy * 1e-3) / 1e9,
+                               "what": "cudaMemcpyAsync of G to HBM, ember_step_dense, state back"}}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

@@ -132,6 +132,18 @@ ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes
 ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *state,
                               float lr, int64_t t, void *stream);
 
+/* The dense step with the gradient in host memory (Grace-Blackwell systems).
+ * Same update as ember_step_dense.  The reduce pass reads G_host directly
+ * over the chip-to-chip link -- no copy engine -- and writes each element to
+ * G_stage (device, V x D fp32, caller-owned) as it goes; the state and apply
+ * passes then read G_stage from HBM.  G_host must be addressable by the GPU:
+ * pinned (cudaHostAlloc / cudaHostRegister), managed or device memory;
+ * unregistered host memory returns EMBER_ERR_INVALID_ARG.  The row-only
+ * variant is not offered here (EMBER_ERR_UNSUPPORTED).  Afterwards G_stage
+ * holds a copy of G. */
+ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G_host, float *G_stage,
+                                        float *state, float lr, int64_t t, void *stream);
+
 /* The dense step for callers that cannot give the library any device
  * memory: hosts whose allocator offers plugins no allocation hook,
  * optimizer loops under a fully reserved memory budget, and code paths

@@ -191,6 +191,56 @@ ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *s
     return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
 }
 
+ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G_host, float *G_stage,
+                                        float *state, float lr, int64_t t, void *stream)
+{
+    if (!h || !W || !G_host || !G_stage || !state)
+        return EMBER_ERR_INVALID_ARG;
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    if (h->hp.variant == EMBER_VARIANT_ROW)
+        return EMBER_ERR_UNSUPPORTED;
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    if (!is_aligned(W, wsz) || !is_aligned(G_host, 4) || !is_aligned(G_stage, 4) || !is_aligned(state, 4))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    // the GPU must be able to address G_host
+    cudaPointerAttributes attr;
+    if (cudaPointerGetAttributes(&attr, G_host) != cudaSuccess) {
+        cudaGetLastError();
+        return EMBER_ERR_INVALID_ARG;
+    }
+    const float *G_dev = static_cast<const float *>(attr.devicePointer);
+    if (attr.type == cudaMemoryTypeUnregistered || !G_dev)
+        return EMBER_ERR_INVALID_ARG;
+
+    DenseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.wbf16 = h->wdtype == EMBER_BF16;
+    a.W = W;
+    a.G = G_dev;
+    a.G_stage = G_stage;
+    a.r = state;
+    a.c = state + h->V;
+    a.beta2 = h->hp.beta2;
+    a.one_minus_beta2 = 1.0 - h->hp.beta2;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.eps = (float)h->hp.eps;
+    a.variant = h->hp.variant;
+    a.ws = h->ws;
+    a.lay = make_layout(h->V, h->D, h->ws_max_N);
+    a.stream = (cudaStream_t)stream;
+    a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && is_aligned(G_dev, 16) &&
+                      is_aligned(G_stage, 16);
+    if (!choose_colmap(h->D, vec4, &a.map))
+        return EMBER_ERR_UNSUPPORTED;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
 ember_status ember_step_sparse(ember_handle *h, void *W, const void *ids, ember_idtype idtype,
                                int64_t N, const float *rows, float *state, float lr, int64_t t,
                                void *stream)

@@ -41,11 +41,15 @@ using namespace dev;
 
 // Pass 1: one read of G.  Template: VEC columns per access, CPT accesses per
 // thread per row, R rows per row group per iteration.
-template <int VEC, int CPT, int R>
+// STAGE: G is read from host memory the GPU can address (over the
+// Grace-Blackwell chip-to-chip link) and every element is also written to
+// G_stage in HBM for the apply pass.
+template <int VEC, int CPT, int R, bool STAGE>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                float *__restrict__ colpart, double *__restrict__ rsum_part,
-               int64_t V, int D, int tpr, double beta2, double one_minus_beta2)
+               int64_t V, int D, int tpr, double beta2, double one_minus_beta2,
+               float *__restrict__ G_stage)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
@@ -88,8 +92,15 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
 #pragma unroll
             for (int c = 0; c < CPT; ++c) {
                 const int col = l + c * tpr;
-                v[k][c] = (i < row1 && col < DV) ? load_g<VEC>(G + i * D + (int64_t)col * VEC)
-                                                 : zero_vec<VEC>();
+                const bool in = i < row1 && col < DV;
+                if constexpr (STAGE) {
+                    const int64_t idx = i * D + (int64_t)col * VEC;
+                    v[k][c] = in ? *reinterpret_cast<const F *>(G + idx) : zero_vec<VEC>();
+                    if (in)
+                        *reinterpret_cast<F *>(G_stage + idx) = v[k][c];
+                } else {
+                    v[k][c] = in ? load_g<VEC>(G + i * D + (int64_t)col * VEC) : zero_vec<VEC>();
+                }
             }
         }
         // squares and per-row partial sums
@@ -621,8 +632,14 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     }
     if (a.trace)
         cudaEventRecord(a.trace[0], a.stream);
-    e = launch_k(k_reduce_dense<VEC, CPT, R1>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                 a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2);
+    if (a.G_stage)
+        e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
+                     a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage);
+    else
+        e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
+                     a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr);
+    // the state and apply passes read the staged copy
+    const float *Gd = a.G_stage ? a.G_stage : a.G;
     if (e != cudaSuccess)
         return e;
     if (a.trace)
@@ -636,11 +653,11 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     const size_t cs_bytes = (size_t)D * sizeof(float);
     if (a.wbf16)
         e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
-                     a.stream, pdl, a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
+                     a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
                      a.eps, a.lr_signed, a.variant);
     else
         e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
-                     a.stream, pdl, a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
+                     a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
                      a.eps, a.lr_signed, a.variant);
     if (e != cudaSuccess)
         return e;

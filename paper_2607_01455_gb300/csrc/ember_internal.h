@@ -103,6 +103,7 @@ struct DenseArgs {
     ColMap map;
     cudaStream_t stream;
     const cudaEvent_t *trace;  // nullptr, or events[0..3] to record at kernel boundaries
+    float *G_stage;            // nullptr, or the HBM copy the reduce pass writes of a host-resident G
 };
 
 cudaError_t launch_dense_step(const DenseArgs &a);

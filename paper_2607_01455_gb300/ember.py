@@ -37,7 +37,7 @@ EXPORTS = (
     "ember_workspace_bytes", "ember_bind_workspace", "ember_step_dense",
     "ember_step_sparse", "ember_get_device_status", "ember_status_string",
     "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
-    "ember_step_dense_noalloc",
+    "ember_step_dense_noalloc", "ember_step_dense_from_host",
 )
 
 
@@ -83,6 +83,7 @@ def lib():
             "ember_set_trace_events": (st, [vp, ctypes.POINTER(vp), ip]),
             "ember_sparse_unique": (st, [vp, vp, ip, i64, vp, vp, vp, vp]),
             "ember_step_dense_noalloc": (st, [vp, vp, vp, vp, flt, i64, vp]),
+            "ember_step_dense_from_host": (st, [vp, vp, vp, vp, vp, flt, i64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -164,6 +165,12 @@ def ember_step_dense_noalloc(h, W, G, state, lr, t, stream=None):
                                           _stream(stream)), "ember_step_dense_noalloc")
 
 
+def ember_step_dense_from_host(h, W, G_host, G_stage, state, lr, t, stream=None):
+    """The dense step reading G from pinned host memory, staging it in G_stage."""
+    _check(lib().ember_step_dense_from_host(h, _addr(W), _addr(G_host), _addr(G_stage), _addr(state),
+                                            lr, t, _stream(stream)), "ember_step_dense_from_host")
+
+
 def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
     _check(lib().ember_step_sparse(h, _addr(W), _addr(ids), idtype, N, _addr(rows), _addr(state),
                                    lr, t, _stream(stream)), "ember_step_sparse")
@@ -224,6 +231,9 @@ class Ember:
 
     def step_dense(self, W, G, lr, t, stream=None):
         ember_step_dense(self.handle, W, G, self.state, lr, t, stream)
+
+    def step_dense_from_host(self, W, G_host, G_stage, lr, t, stream=None):
+        ember_step_dense_from_host(self.handle, W, G_host, G_stage, self.state, lr, t, stream)
 
     def step_sparse(self, W, ids, rows, lr, t, stream=None):
         import torch

@@ -100,6 +100,18 @@ def test_create_rejects(kw, status):
     assert ex.value.status == status
 
 
+def test_from_host_refuses_row_only_variant():
+    hp = E.ember_hparams_default()
+    hp.variant = E.EMBER_VARIANT_ROW
+    h = E.ember_create(16, 8, hp)
+    try:
+        fake = 1 << 20
+        assert E.lib().ember_step_dense_from_host(h, fake, fake, fake, fake, 1e-3, 1, None) == \
+            E.EMBER_ERR_UNSUPPORTED
+    finally:
+        E.ember_destroy(h)
+
+
 def test_create_accepts_limits():
     for V, D in [(1, 8192), (3, 2048), (2, 2047), (1, 3)]:
         E.ember_destroy(E.ember_create(V, D))
@@ -131,7 +143,14 @@ def test_step_and_bind_reject_on_host():
         assert lib.ember_step_sparse(h, fake, None, 0, 4, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_INVALID_ARG
         assert lib.ember_step_sparse(h, fake, fake, 5, 4, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_DTYPE
         assert lib.ember_step_sparse(h, fake, fake, 1, 4, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
-        assert lib.ember_get_device_status(h, None) == E.EMBER_ERR_WORKSPACE
+        # dense step from host memory: rejected before any CUDA call
+        fh = lib.ember_step_dense_from_host
+        assert fh(h, fake, None, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert fh(h, fake, fake, None, fake, 1e-3, 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert fh(h, fake, fake, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
+        assert fh(h, fake, fake + 2, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_ALIGNMENT
+        assert fh(h, fake, fake, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
+        assert E.lib().ember_get_device_status(h, None) == E.EMBER_ERR_WORKSPACE
         assert lib.ember_get_device_status(None, None) == E.EMBER_ERR_INVALID_ARG
     finally:
         E.ember_destroy(h)

@@ -223,3 +223,35 @@ def test_dense_graph_capture_matches_eager(cuda_device):
     torch.cuda.synchronize()
     assert torch.equal(W1.view(torch.int16), W2.view(torch.int16))
     assert torch.equal(e1.state, e2.state)
+
+
+@pytest.mark.parametrize("V,D,wdtype", [(3001, 1024, "bf16"), (2000, 8192, "bf16"), (513, 203, "f32")])
+def test_step_from_host_matches_device_step(cuda_device, V, D, wdtype):
+    """The gradient read from pinned host memory (and staged in HBM by the
+    reduce pass) gives the same W and state, bit for bit, as the step on a
+    device-resident gradient; the stage holds an exact copy of G."""
+    a, b = make(V, D, wdtype), make(V, D, wdtype)
+    Wa = rand_w(V, D, wdtype, cuda_device)
+    Wb = Wa.clone()
+    stage = torch.empty(V, D, device=cuda_device)
+    for t in (1, 2):
+        G = rand_grad(V, D, t, cuda_device, seed=D)
+        Gh = G.cpu().pin_memory()
+        a.step_dense(Wa, G, 1e-3, t)
+        b.step_dense_from_host(Wb, Gh, stage, 1e-3, t)
+        torch.cuda.synchronize()
+        assert torch.equal(stage, G)
+        assert torch.equal(Wa.view(torch.int16) if wdtype == "bf16" else Wa,
+                           Wb.view(torch.int16) if wdtype == "bf16" else Wb)
+        assert torch.equal(a.state, b.state)
+
+
+def test_step_from_host_refuses_unregistered_memory(cuda_device):
+    V, D = 64, 32
+    emb = make(V, D, "bf16")
+    W = rand_w(V, D, "bf16", cuda_device)
+    pageable = np.zeros((V, D), np.float32)
+    stage = torch.empty(V, D, device=cuda_device)
+    with pytest.raises(EmberError) as ex:
+        emb.step_dense_from_host(W, pageable.ctypes.data, stage, 1e-3, 1)
+    assert ex.value.status == 1  # EMBER_ERR_INVALID_ARG
