@@ -119,8 +119,22 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
            for i, name in enumerate(SPARSE_KERNELS)}
     ms = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain)
     ms_traced = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in traced) / len(traced)
+    # the same step replayed from a CUDA graph (how a training loop would run it)
+    side = torch.cuda.Stream(dev)
+    side.wait_stream(torch.cuda.current_stream(dev))
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=side):
+        emb.step_sparse(W, ids, rows, wl.lr, t + 1, stream=side)
+    gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for k in range(steps):
+        flush.zero_()
+        gev[k][0].record()
+        graph.replay()
+        gev[k][1].record()
+    torch.cuda.synchronize()
+    ms_graph = sum(a.elapsed_time(b) for a, b in gev) / steps
     B = sparse_bytes(wl, U)
-    return {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "unique_ids": U,
+    return {"workload": wl.name, "ms_per_step_graph": ms_graph, "V": wl.V, "D": wl.D, "N": wl.N, "unique_ids": U,
             "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
             "algorithmic_bytes": B, "touched_params_per_s": U * wl.D / (ms * 1e-3),
             "occurrence_params_per_s": wl.N * wl.D / (ms * 1e-3),

@@ -45,7 +45,7 @@ def rand_w(V, D, wdtype, device, seed=0):
 SHAPES = [
     (1, 1), (1, 4), (2, 3), (7, 5), (37, 64), (303, 96), (304, 128), (305, 132),
     (1000, 200), (1000, 203), (3001, 256), (777, 1028), (2049, 896), (513, 2048),
-    (64, 2047), (150, 4096), (40, 8192),
+    (64, 2047), (150, 4096), (40, 8192), (2, 1), (1000, 33), (7, 127),
 ]
 
 
