@@ -393,9 +393,12 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
     using F = typename Vec<VEC>::F;
     constexpr int R = 8;  // rows in flight per thread
     constexpr int kWarps = kThreads / 32;
-    constexpr int kFin = 32;  // completed runs buffered before their g^2 sums are written
+    constexpr int kFin = 128;  // completed runs buffered before their g^2 sums are written
+    constexpr int kIdxWindow = 1024;
     __shared__ float rp[kFin][kWarps];
     __shared__ int fin[kFin];
+    __shared__ int sperm[kIdxWindow];
+    __shared__ int sseg[kIdxWindow];
     const int DV = D / VEC;
     const int sigma = blockIdx.x % NS;
     const int w = blockIdx.x / NS;
@@ -482,34 +485,45 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                 *reinterpret_cast<F *>(carry + ((int64_t)2 * w + which) * D + (int64_t)col * VEC) = acc;
             }
         };
-        for (int pb = p0; pb < p1; pb += R) {
-            F v[R];
-            int uu[R];
-#pragma unroll
-            for (int k = 0; k < R; ++k) {
-                const int p = pb + k;
-                uu[k] = -1;
-                v[k] = zero_vec<VEC>();
-                if (p < p1) {
-                    uu[k] = segidx[p];
-                    if (active)
-                        v[k] = load_g<VEC>(rows + (int64_t)perm[p] * D + (int64_t)col * VEC);
-                }
+        // The range's occurrence and run indices go to shared memory a
+        // window at a time, so each batch of rows costs one trip to HBM.
+        for (int wb = p0; wb < p1; wb += kIdxWindow) {
+            const int we = (wb + kIdxWindow < p1) ? wb + kIdxWindow : p1;
+            __syncthreads();  // the previous window's indices are no longer read
+            for (int p = wb + threadIdx.x; p < we; p += kThreads) {
+                sperm[p - wb] = perm[p];
+                sseg[p - wb] = segidx[p];
             }
+            __syncthreads();
+            for (int pb = wb; pb < we; pb += R) {
+                F v[R];
+                int uu[R];
 #pragma unroll
-            for (int k = 0; k < R; ++k) {
-                if (uu[k] < 0)
-                    break;
-                if (uu[k] != cur) {
-                    flush(cur);
-                    acc = zero_vec<VEC>();
-                    cur = uu[k];
-                    len = 0;
+                for (int k = 0; k < R; ++k) {
+                    const int p = pb + k;
+                    uu[k] = -1;
+                    v[k] = zero_vec<VEC>();
+                    if (p < we) {
+                        uu[k] = sseg[p - wb];
+                        if (active)
+                            v[k] = load_g<VEC>(rows + (int64_t)sperm[p - wb] * D + (int64_t)col * VEC);
+                    }
                 }
-                ++len;
 #pragma unroll
-                for (int e = 0; e < VEC; ++e)
-                    set_comp(acc, e, comp(acc, e) + comp(v[k], e));
+                for (int k = 0; k < R; ++k) {
+                    if (uu[k] < 0)
+                        break;
+                    if (uu[k] != cur) {
+                        flush(cur);
+                        acc = zero_vec<VEC>();
+                        cur = uu[k];
+                        len = 0;
+                    }
+                    ++len;
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e)
+                        set_comp(acc, e, comp(acc, e) + comp(v[k], e));
+                }
             }
         }
         flush(cur);
