@@ -11,7 +11,9 @@ Arrays are numpy and are updated in place:
 * ``W``: V x D, ``np.float32`` or bfloat16 bit patterns as ``np.uint16``;
 * ``G``: V x D ``np.float32``; ``rows``: N x D ``np.float32``;
 * ``ids``: N ``np.int64`` token ids;
-* ``r``: V ``np.float32``; ``c``: D ``np.float32`` (the whole optimizer state).
+* ``r``: V ``np.float32``; ``c``: D ``np.float32`` (the whole optimizer state);
+* ``dlogits``: T x V and ``hidden``: T x D, bfloat16 bit patterns (``np.uint16``),
+  the two factors of an LM head's gradient.
 
 Parity status: every function is pinned by tests/test_oracle_pins.py except
 the behaviour of gradients so small that g^2 or the fp32 state underflows,
@@ -46,6 +48,8 @@ def _load():
         lib.ember_oracle_round_bf16.restype = None
         lib.ember_oracle_bf16_to_double.argtypes = [i64, vp, vp]
         lib.ember_oracle_bf16_to_double.restype = None
+        lib.ember_oracle_lmhead_grad.argtypes = [i64, i64, i64, vp, vp, i64, vp, vp, vp]
+        lib.ember_oracle_lmhead_grad.restype = ip
         _lib = lib
     return _lib
 
@@ -137,3 +141,31 @@ def bf16_to_float64(bits):
     out = np.zeros(bits.shape, np.float64)
     _load().ember_oracle_bf16_to_double(bits.size, _ptr(bits), _ptr(out))
     return out
+
+
+def lmhead_grad(dlogits, hidden, rows=None):
+    """The LM-head gradient G = dlogits^T hidden (appendix "Decomposing the
+    Squared Gradient": a sum over tokens of the outer product of the softmax
+    error and the hidden state), in fp64, summed in token order.
+
+    ``dlogits`` (T x V) and ``hidden`` (T x D) are bfloat16 bit patterns.
+    ``rows``: the row indices v to compute (default: all).  Returns
+    ``(G, absG)``, both len(rows) x D float64; ``absG`` is sum_t |delta h|."""
+    dlogits = np.ascontiguousarray(dlogits, dtype=np.uint16)
+    hidden = np.ascontiguousarray(hidden, dtype=np.uint16)
+    if dlogits.ndim != 2 or hidden.ndim != 2 or dlogits.shape[0] != hidden.shape[0]:
+        raise ValueError("dlogits must be T x V and hidden T x D")
+    T, V = dlogits.shape
+    D = hidden.shape[1]
+    if rows is None:
+        nrows, rp = V, None
+    else:
+        rows = np.ascontiguousarray(rows, dtype=np.int64)
+        nrows, rp = rows.shape[0], _ptr(rows)
+    G = np.zeros((nrows, D), np.float64)
+    A = np.zeros((nrows, D), np.float64)
+    rc = _load().ember_oracle_lmhead_grad(T, V, D, _ptr(dlogits), _ptr(hidden), nrows, rp,
+                                           _ptr(G), _ptr(A))
+    if rc != 0:
+        raise ValueError(f"oracle LM-head gradient rejected its arguments (code {rc})")
+    return G, A

@@ -290,3 +290,61 @@ int64_t ember_oracle_dedup(int64_t N, const int64_t *ids, int64_t V,
     free(tmp);
     return U;
 }
+
+/* ------------------------------------------------------------------ */
+/* LM-head gradient, the step that produces G for an output head       */
+/* (appendix "Decomposing the Squared Gradient"): token t contributes  */
+/* the outer product of its output-side error delta_t (V values, the   */
+/* softmax error) and its hidden state h_t (D values); the batch        */
+/* gradient is the sum over the T tokens, G = dlogits^T H, i.e.        */
+/*   G[v][d] = sum_t dlogits[t][v] * hidden[t][d].                     */
+/* Inputs are bfloat16 bit patterns, row-major T x V and T x D.  Each  */
+/* product and the sum over t (in token order) are taken in fp64.      */
+/* rows: the nrows row indices v to compute (NULL: all V rows, in      */
+/* order); G and absG receive nrows x D values.  absG (optional) gets   */
+/* sum_t |dlogits[t][v] hidden[t][d]|, the scale against which the    */
+/* rounding of any other summation order is bounded.                   */
+/* ------------------------------------------------------------------ */
+
+int ember_oracle_lmhead_grad(int64_t T, int64_t V, int64_t D,
+                             const uint16_t *dlogits, const uint16_t *hidden,
+                             int64_t nrows, const int64_t *rows,
+                             double *G, double *absG)
+{
+    if (T < 0 || V < 1 || D < 1 || !G || (T > 0 && (!dlogits || !hidden)))
+        return ORC_EINVAL;
+    if (!rows)
+        nrows = V;
+    if (nrows < 0)
+        return ORC_EINVAL;
+    double *hrow = (double *)malloc((size_t)D * sizeof(double));
+    if (!hrow)
+        return ORC_ENOMEM;
+    for (int64_t q = 0; q < nrows; ++q) {
+        int64_t v = rows ? rows[q] : q;
+        if (v < 0 || v >= V) {
+            free(hrow);
+            return ORC_EINVAL;
+        }
+        double *out = G + q * D;
+        double *aout = absG ? absG + q * D : NULL;
+        for (int64_t d = 0; d < D; ++d) {
+            out[d] = 0.0;
+            if (aout)
+                aout[d] = 0.0;
+        }
+        for (int64_t t = 0; t < T; ++t) {
+            double delta = bf16_bits_to_double(dlogits[t * V + v]);
+            for (int64_t d = 0; d < D; ++d)
+                hrow[d] = bf16_bits_to_double(hidden[t * D + d]);
+            for (int64_t d = 0; d < D; ++d) {
+                double p = delta * hrow[d];
+                out[d] += p;
+                if (aout)
+                    aout[d] += fabs(p);
+            }
+        }
+    }
+    free(hrow);
+    return ORC_OK;
+}

@@ -38,6 +38,12 @@ MUTANTS = {
                                 "Gd[id * D + j] = (double)rows[k * D + j];"),
     "bf16 ties away from zero": ("double q = rint(a / quantum);", "double q = round(a / quantum);"),
     "bf16 subnormals dropped": ("if (lead < -126)", "if (lead < -140)"),
+    "LM-head gradient drops the last token": ("for (int64_t t = 0; t < T; ++t) {",
+                                              "for (int64_t t = 0; t < T - 1; ++t) {"),
+    "LM-head hidden state of the wrong token": ("hrow[d] = bf16_bits_to_double(hidden[t * D + d]);",
+                                                "hrow[d] = bf16_bits_to_double(hidden[((t + 1) % T) * D + d]);"),
+    "LM-head error of the neighbouring row": ("double delta = bf16_bits_to_double(dlogits[t * V + v]);",
+                                              "double delta = bf16_bits_to_double(dlogits[t * V + (v + 1) % V]);"),
 }
 
 

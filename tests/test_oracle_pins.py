@@ -443,3 +443,82 @@ def test_paper_state_sizes_follow_from_v_plus_d():
         assert _in_unit(adamw_bytes, aunit) == pytest.approx(aval, rel=0.01), e["model"]
         if "ratio" in e:
             assert adamw_bytes / ember_bytes == pytest.approx(e["ratio"][0], rel=0.02), e["model"]
+
+
+# --------------------------------------------------------------------------
+# LM-head gradient, the producer of G for an output head (appendix
+# "Decomposing the Squared Gradient": per token the outer product of the
+# softmax error and the hidden state, summed over the batch).
+# --------------------------------------------------------------------------
+
+def _bf16_bits(rng, shape, lo=-8, hi=2):
+    """Random finite bfloat16 bit patterns with exponents in [lo, hi)."""
+    mant = rng.integers(0, 128, size=shape).astype(np.uint32)
+    expo = (rng.integers(lo, hi, size=shape) + 127).astype(np.uint32)
+    sign = rng.integers(0, 2, size=shape).astype(np.uint32)
+    return ((sign << 15) | (expo << 7) | mant).astype(np.uint16)
+
+
+def test_lmhead_grad_matches_exact_rational_sum():
+    """Brute force in exact rationals: G[v][d] = sum_t delta[t][v] h[t][d].  The
+    fp64 result may differ from the exact sum only by the rounding of T - 1
+    additions of exactly representable products (bf16 x bf16 fits in 16 bits)."""
+    from fractions import Fraction
+    rng = np.random.default_rng(11)
+    T, V, D = 6, 5, 7
+    dl = _bf16_bits(rng, (T, V))
+    hd = _bf16_bits(rng, (T, D))
+    G, A = oracle.lmhead_grad(dl, hd)
+    dv = oracle.bf16_to_float64(dl)
+    hv = oracle.bf16_to_float64(hd)
+    for v in range(V):
+        for d in range(D):
+            exact = sum(Fraction(dv[t, v]) * Fraction(hv[t, d]) for t in range(T))
+            absum = sum(abs(Fraction(dv[t, v]) * Fraction(hv[t, d])) for t in range(T))
+            assert abs(Fraction(G[v, d]) - exact) <= Fraction(T) * Fraction(2) ** -53 * absum
+            assert A[v, d] == pytest.approx(float(absum), rel=1e-15)
+
+
+def test_lmhead_grad_one_hot_errors_gather_hidden_rows():
+    """With delta_t = -e_{y_t} (a softmax error whose model probabilities are
+    all zero), row v of G is minus the sum of the hidden states of the tokens
+    whose target is v; rows of tokens never targeted are exactly zero."""
+    rng = np.random.default_rng(12)
+    T, V, D = 40, 9, 16
+    y = rng.integers(0, V - 2, size=T)  # the last two rows are never targeted
+    dl = np.zeros((T, V), np.uint16)
+    dl[np.arange(T), y] = 0xBF80  # bfloat16 -1.0
+    hd = _bf16_bits(rng, (T, D), lo=-4, hi=1)
+    G, _ = oracle.lmhead_grad(dl, hd)
+    want = np.zeros((V, D))
+    np.add.at(want, y, -oracle.bf16_to_float64(hd))
+    np.testing.assert_array_equal(G, want)
+    assert not G[V - 2:].any()
+
+
+def test_lmhead_grad_single_token_is_outer_product():
+    rng = np.random.default_rng(13)
+    dl = _bf16_bits(rng, (1, 11))
+    hd = _bf16_bits(rng, (1, 6))
+    G, A = oracle.lmhead_grad(dl, hd)
+    outer = np.outer(oracle.bf16_to_float64(dl[0]), oracle.bf16_to_float64(hd[0]))
+    np.testing.assert_array_equal(G, outer)
+    np.testing.assert_array_equal(A, np.abs(outer))
+
+
+def test_lmhead_grad_roles_of_the_factors_and_row_selection():
+    """Swapping the two factors transposes G (each element is the same sum in
+    the same token order); a selected row equals that row of the full G."""
+    rng = np.random.default_rng(14)
+    T, V, D = 13, 10, 7
+    dl = _bf16_bits(rng, (T, V))
+    hd = _bf16_bits(rng, (T, D))
+    G, _ = oracle.lmhead_grad(dl, hd)
+    Gt, _ = oracle.lmhead_grad(hd, dl)
+    np.testing.assert_array_equal(Gt, G.T)
+    rows = np.array([9, 0, 4])
+    Gs, _ = oracle.lmhead_grad(dl, hd, rows=rows)
+    np.testing.assert_array_equal(Gs, G[rows])
+    # matmul of the exact factors in fp64 agrees to rounding
+    ref = oracle.bf16_to_float64(dl).T @ oracle.bf16_to_float64(hd)
+    np.testing.assert_allclose(G, ref, rtol=0, atol=1e-12 * np.abs(ref).max())
