@@ -164,6 +164,39 @@ ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G
 ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const float *G, float *state,
                                       float lr, int64_t t, void *stream);
 
+/* The gradient of an LM head (output embedding) W = V x D, formed on the
+ * tensor cores: G = dlogits^T hidden, i.e. G[v][d] = sum_t dlogits[t][v]
+ * hidden[t][d], the sum over the T tokens of the outer product of each
+ * token's output-side error (softmax minus one-hot) and its hidden state
+ * (appendix "Decomposing the Squared Gradient").  bf16 products, fp32
+ * accumulation.
+ *   dlogits: T x V bfloat16, row-major, device (any 1/T scaling applied).
+ *   hidden:  T x D bfloat16, row-major, device.
+ *   T:       tokens, 1 <= T <= 2^31 - 1.
+ *   G:       V x D fp32, row-major, device, written (caller-owned).
+ * Requires V % 8 == 0 and D % 8 == 0 (rows of dlogits and hidden a multiple
+ * of 16 bytes; EMBER_ERR_UNSUPPORTED otherwise) and 16-byte aligned
+ * dlogits, hidden and G (EMBER_ERR_ALIGNMENT).  Uses the bound workspace;
+ * the optimizer state is untouched.  A bounded wait inside the kernel that
+ * gives up sets EMBER_ERR_TIMEOUT in the device flag. */
+ember_status ember_lmhead_grad(ember_handle *h, const void *dlogits, const void *hidden, int64_t T,
+                               float *G, void *stream);
+
+/* One dense Ember step (Algorithm 1) of an LM head whose gradient is formed
+ * here: G = dlogits^T hidden exactly as ember_lmhead_grad (G is written, the
+ * same bits), then the step of ember_step_dense on that G.  The kernel that
+ * forms G also writes, from the registers that hold each finished 128 x 256
+ * tile, the tile's sums of g^2 along its rows and along its columns (the
+ * fused deterministic reduction of Section 2.3, moved into the producer of
+ * G); the state pass finishes those sums in a fixed order and the apply pass
+ * reads G once, so the step moves 8VD + 2wVD bytes of G and W instead of
+ * 12VD (bf16 W).  Results are bit-identical from run to run; they match
+ * ember_step_dense on the same G to rounding (the sums of g^2 are grouped
+ * differently).  Every variant is accepted.  Requirements: those of
+ * ember_lmhead_grad and of ember_step_dense. */
+ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, const void *hidden,
+                               int64_t T, float *G, float *state, float lr, int64_t t, void *stream);
+
 /* One sparse Ember step (Section 2.2) at step number t >= 1.
  *   ids:   N token ids of type idtype (duplicates allowed, any order).
  *   rows:  N x D fp32, row k is the gradient contribution of occurrence k

@@ -46,6 +46,8 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
         L.sp_bounds = take(sizeof(int32_t) * ((size_t)kSparseCtas + 1));
         L.sp_rows = take(sizeof(float) * N * (size_t)D);
     }
+    L.lm_colpart = take(sizeof(float) * (size_t)lmhead_row_blocks(V) * (size_t)D);
+    L.lm_rowpart = take(sizeof(float) * (size_t)lmhead_col_blocks(D) * (size_t)V);
     L.total = off;
     return L;
 }
@@ -236,6 +238,77 @@ ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G
     a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
     const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && is_aligned(G_dev, 16) &&
                       is_aligned(G_stage, 16);
+    if (!choose_colmap(h->D, vec4, &a.map))
+        return EMBER_ERR_UNSUPPORTED;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+static ember_status check_lmhead(const ember_handle *h, const void *dlogits, const void *hidden, int64_t T,
+                                 const float *G)
+{
+    if (!dlogits || !hidden || !G || T < 1 || T > INT32_MAX)
+        return EMBER_ERR_INVALID_ARG;
+    if (h->V % 8 != 0 || h->D % 8 != 0 || h->V > INT32_MAX)
+        return EMBER_ERR_UNSUPPORTED;
+    if (!is_aligned(dlogits, 16) || !is_aligned(hidden, 16) || !is_aligned(G, 16))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    return EMBER_OK;
+}
+
+ember_status ember_lmhead_grad(ember_handle *h, const void *dlogits, const void *hidden, int64_t T, float *G,
+                               void *stream)
+{
+    if (!h)
+        return EMBER_ERR_INVALID_ARG;
+    const ember_status st = check_lmhead(h, dlogits, hidden, T, G);
+    if (st != EMBER_OK)
+        return st;
+    const Layout L = make_layout(h->V, h->D, h->ws_max_N);
+    LmArgs lm{h->V, h->D, T, dlogits, hidden, G};
+    DevScalars *sc = reinterpret_cast<DevScalars *>(h->ws + L.scalars);
+    const cudaError_t e = launch_lmhead_grad(lm, reinterpret_cast<float *>(h->ws + L.lm_colpart),
+                                             reinterpret_cast<float *>(h->ws + L.lm_rowpart), &sc->flags,
+                                             (cudaStream_t)stream);
+    return e == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, const void *hidden, int64_t T,
+                               float *G, float *state, float lr, int64_t t, void *stream)
+{
+    if (!h || !W || !state)
+        return EMBER_ERR_INVALID_ARG;
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    const ember_status st = check_lmhead(h, dlogits, hidden, T, G);
+    if (st != EMBER_OK)
+        return st;
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    if (!is_aligned(W, wsz) || !is_aligned(state, 4))
+        return EMBER_ERR_ALIGNMENT;
+
+    LmArgs lm{h->V, h->D, T, dlogits, hidden, G};
+    DenseArgs a{};
+    a.V = h->V;
+    a.D = h->D;
+    a.wbf16 = h->wdtype == EMBER_BF16;
+    a.W = W;
+    a.G = G;
+    a.r = state;
+    a.c = state + h->V;
+    a.beta2 = h->hp.beta2;
+    a.one_minus_beta2 = 1.0 - h->hp.beta2;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.eps = (float)h->hp.eps;
+    a.variant = h->hp.variant;
+    a.ws = h->ws;
+    a.lay = make_layout(h->V, h->D, h->ws_max_N);
+    a.stream = (cudaStream_t)stream;
+    a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    a.lm = &lm;
+    const bool vec4 = is_aligned(W, 4 * wsz);  // D % 8 == 0 and G 16-byte aligned already
     if (!choose_colmap(h->D, vec4, &a.map))
         return EMBER_ERR_UNSUPPORTED;
     return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;

@@ -282,9 +282,15 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
         double rsum = 0.0;
         for (int64_t i = (int64_t)rb * kStateThreads + threadIdx.x; i < V;
              i += (int64_t)rowp.nrow_ctas * kStateThreads) {
-            const int sl = rowp.slot[i];
             double mean_row = 0.0;
-            if (sl) {
+            if (rowp.slot == nullptr) {
+                // every row: per-column-block sums, slice-major, in block order
+                float tot = 0.f;
+#pragma unroll 8
+                for (int k = 0; k < rowp.nslices; ++k)
+                    tot += __ldcg(rowp.rowpart + (int64_t)k * V + i);
+                mean_row = (double)tot / (double)D;
+            } else if (const int sl = rowp.slot[i]) {
                 const int64_t u = sl - 1;
                 float tot = 0.f;
                 for (int k = 0; k < rowp.nslices; ++k)
@@ -603,7 +609,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     // dependent launch.
     const bool pdl = (a.trace == nullptr);
     cudaError_t e;
-    if (a.variant == EMBER_VARIANT_ROW) {
+    if (a.variant == EMBER_VARIANT_ROW && !a.lm) {
         // one pass over G and W, then the column state; no apply pass
         constexpr int RR = (4 / CPT) < 1 ? 1 : (4 / CPT);
         if (a.trace)
@@ -630,24 +636,45 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         }
         return cudaGetLastError();
     }
-    if (a.trace)
-        cudaEventRecord(a.trace[0], a.stream);
-    if (a.G_stage)
-        e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                     a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage);
-    else
-        e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                     a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr);
-    // the state and apply passes read the staged copy
-    const float *Gd = a.G_stage ? a.G_stage : a.G;
-    if (e != cudaSuccess)
-        return e;
-    if (a.trace)
-        cudaEventRecord(a.trace[1], a.stream);
-    e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                     a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
-    if (e != cudaSuccess)
-        return e;
+    if (a.lm) {
+        // G comes from the LM-head kernel, which also leaves the sums of g^2
+        // per 128-row block (columns) and per 256-column block (rows); the
+        // state pass finishes both, then the apply pass reads G once.
+        float *lm_col = reinterpret_cast<float *>(a.ws + a.lay.lm_colpart);
+        float *lm_row = reinterpret_cast<float *>(a.ws + a.lay.lm_rowpart);
+        if (a.trace)
+            cudaEventRecord(a.trace[0], a.stream);
+        e = launch_lmhead_grad(*a.lm, lm_col, lm_row, &sc->flags, a.stream);
+        if (e != cudaSuccess)
+            return e;
+        if (a.trace)
+            cudaEventRecord(a.trace[1], a.stream);
+        const int nrow_ctas = kSms;
+        e = launch_state(lm_col, lmhead_row_blocks(a.V), rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D,
+                         a.beta2, a.one_minus_beta2, a.inv_bc, a.stream, pdl, a.r, nullptr, lm_row,
+                         lmhead_col_blocks(a.D), nrow_ctas);
+        if (e != cudaSuccess)
+            return e;
+    } else {
+        if (a.trace)
+            cudaEventRecord(a.trace[0], a.stream);
+        if (a.G_stage)
+            e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
+                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage);
+        else
+            e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
+                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr);
+        if (e != cudaSuccess)
+            return e;
+        if (a.trace)
+            cudaEventRecord(a.trace[1], a.stream);
+        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        if (e != cudaSuccess)
+            return e;
+    }
+    // the apply pass reads the staged copy, or the G the LM-head kernel wrote
+    const float *Gd = a.lm ? a.lm->G : a.G_stage ? a.G_stage : a.G;
     if (a.trace)
         cudaEventRecord(a.trace[2], a.stream);
     const size_t cs_bytes = (size_t)D * sizeof(float);

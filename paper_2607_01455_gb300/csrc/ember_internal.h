@@ -72,6 +72,9 @@ struct Layout {
     size_t sp_carry;    // float[2 * kSparseCtas * D]  partial sums of runs cut by worker ranges
     size_t sp_bounds;   // int32[kSparseCtas + 1]  first sorted position of each worker range
     size_t sp_rows;     // float[N * D]  summed gradient row of each distinct id seen twice or more
+    // LM-head step (the gradient formed here on the tensor cores)
+    size_t lm_colpart;  // float[ceil(V/128) * D]  sums of g^2 over each 128-row block
+    size_t lm_rowpart;  // float[ceil(D/256) * V]  sums of g^2 over each 256-column block
     size_t total;
 };
 
@@ -86,6 +89,21 @@ struct ColMap {
 };
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m);
+
+// LM-head gradient G = dlogits^T hidden (T tokens, bf16 inputs, fp32 G).
+struct LmArgs {
+    int64_t V, D, T;
+    const void *dlogits;  // T x V bf16
+    const void *hidden;   // T x D bf16
+    float *G;             // V x D fp32, written
+};
+
+int lmhead_row_blocks(int64_t V);
+int lmhead_col_blocks(int64_t D);
+// Forms G and the per-tile sums of g^2 (colpart: [row blocks][D], rowpart:
+// [column blocks][V]); a bounded wait that gives up sets kFlagTimeout in *flags.
+cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
+                               cudaStream_t stream);
 
 struct DenseArgs {
     int64_t V, D;
@@ -104,12 +122,15 @@ struct DenseArgs {
     cudaStream_t stream;
     const cudaEvent_t *trace;  // nullptr, or events[0..3] to record at kernel boundaries
     float *G_stage;            // nullptr, or the HBM copy the reduce pass writes of a host-resident G
+    const LmArgs *lm;          // nullptr, or: G is formed by the LM-head kernel instead of read
 };
 
 cudaError_t launch_dense_step(const DenseArgs &a);
 
-// Column EMA and normaliser; with nrow_ctas > 0 the same launch also runs the
-// sparse step's row pass (r for all V rows from the per-slice sums of g^2).
+// Column EMA and normaliser; with nrow_ctas > 0 the same launch also runs a
+// row pass: r for all V rows from per-slice sums of g^2, taken from
+// rowpart[slot[i]-1][nslices] for the sparse step (rows with slot 0 saw no
+// gradient) or, with slot == nullptr, from rowpart[nslices][V] for every row.
 cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, int nrsum, float *c,
                          double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
                          double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl,

@@ -1,0 +1,521 @@
+// LM-head gradient on the tensor cores, with the Ember statistics in the
+// epilogue.
+//
+// For an output head the per-token gradient is the outer product of the
+// token's softmax error delta_t (V values) and its hidden state h_t (D
+// values), and the batch gradient is their sum over the T tokens:
+//     G = dlogits^T H,   G[v][d] = sum_t dlogits[t][v] H[t][d]
+// (appendix "Decomposing the Squared Gradient").  Algorithm 1 then needs the
+// sums of g^2 along every row and every column of G.  This kernel forms G
+// tile by tile with tcgen05.mma (bf16 in, fp32 accumulate in tensor memory)
+// and, while a finished tile is in registers for its store, also writes the
+// tile's per-row and per-column sums of g^2.  The optimizer step then skips
+// its reduction pass (one 4VD-byte read of G) and goes straight to the state
+// and apply passes: the fused deterministic reduction of Section 2.3, moved
+// into the producer of G.
+//
+// Tiles: 128 rows of G (vocabulary) x 256 columns (features), the largest
+// single-CTA tcgen05 shape; 64 tokens per pipeline stage, 4 stages.  Both
+// operands are "MN-major" in memory (dlogits is T x V and H is T x D, row-
+// major, so for fixed token the tile's rows, resp. columns, are contiguous):
+// each stage is loaded by TMA as 64-wide boxes with the 128-byte swizzle and
+// described to the MMA as MN-major, swizzled, 8 KiB between 64-element
+// blocks and 1 KiB between 8-token groups.
+//
+// Warp roles (256 threads, one CTA per SM, persistent over tiles):
+//   warp 0   one thread issues the TMA loads of every stage
+//   warp 1   allocates 512 tensor-memory columns (two 128 x 256 fp32
+//            accumulators, so the epilogue of one tile overlaps the MMAs of
+//            the next); one thread issues the MMAs
+//   warps 4-7  epilogue: warp 4+q reads accumulator lanes 32q..32q+31 (rows
+//            of the tile), stores G, and forms the sums of g^2
+//
+// Determinism: every output element of G, of the per-tile row sums and of
+// the per-tile column sums is produced by exactly one tile, in a fixed
+// order; nothing is accumulated across CTAs here.  The state pass sums the
+// per-tile partials in a fixed order.
+//
+// Waits on mbarriers are bounded (kWaitNs of wall time); a wait that gives up
+// sets the sticky timeout flag, stops every role, lets the copies and MMAs
+// already issued finish, frees the tensor memory and returns.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <mutex>
+
+#include "ember_device.cuh"
+#include "ember_internal.h"
+
+namespace ember {
+namespace {
+
+constexpr int kBM = 128;                    // tile rows (UMMA M)
+constexpr int kBN = 256;                    // tile columns (UMMA N)
+constexpr int kBK = 64;                     // tokens per stage
+constexpr int kUK = 16;                     // K of one kind::f16 MMA
+constexpr int kStages = 4;
+constexpr int kBox = 64;                    // TMA box: 64 bf16 = 128 bytes, the swizzle span
+constexpr int kABytes = kBM * kBK * 2;      // 16 KiB
+constexpr int kBBytes = kBN * kBK * 2;      // 32 KiB
+constexpr int kStageBytes = kABytes + kBBytes;
+constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 8 KiB
+constexpr int kAccCols = kBN;               // fp32 accumulator columns per tile
+constexpr int kTmemCols = 2 * kAccCols;     // two accumulators
+constexpr int kLmThreads = 256;
+constexpr int kEpiWarp0 = 4;
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
+
+// Shared memory: stages (1 KiB aligned for the swizzle), then barriers.
+struct LmSmemTail {
+    uint64_t full[kStages];    // TMA bytes landed
+    uint64_t empty[kStages];   // MMAs of the stage done
+    uint64_t tfull[2];         // accumulator ready for the epilogue
+    uint64_t tempty[2];        // accumulator drained by the epilogue
+    uint64_t drain;            // every MMA issued has completed
+    uint32_t tmem_base;
+    int abort;
+    float xch[2][4][32];       // per-warp column sums, double-buffered
+};
+constexpr size_t kLmSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(LmSmemTail);
+
+__device__ __forceinline__ uint32_t smem_addr(const void *p)
+{
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ uint64_t now_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
+{
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase of parity `parity` of `bar` to complete.  Gives up when
+// another role has aborted or after kWaitNs; returns false then.
+__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort)
+{
+    if (mbar_test(bar, parity))
+        return true;
+    const uint64_t t0 = now_ns();
+    for (uint32_t k = 1;; ++k) {
+        if (mbar_test(bar, parity))
+            return true;
+        if ((k & 63u) == 0) {
+            if (*abort)
+                return false;
+            if (now_ns() - t0 > kWaitNs)
+                return false;
+        }
+    }
+}
+
+// Same, for teardown: no abort check, only the time limit.
+__device__ bool mbar_wait_final(uint32_t bar, uint32_t parity)
+{
+    const uint64_t t0 = now_ns();
+    while (!mbar_test(bar, parity))
+        if (now_ns() - t0 > kWaitNs)
+            return false;
+    return true;
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                            uint32_t bar)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor of tcgen05.mma for an MN-major operand
+// with the 128-byte swizzle: start address, 8 KiB between 64-element blocks
+// along M (or N) ("leading" offset), 1 KiB between groups of 8 rows along K
+// ("stride" offset), descriptor version 1, swizzle mode 2 (128 bytes).
+__device__ __forceinline__ uint64_t mn_major_sw128_desc(uint32_t saddr)
+{
+    uint64_t d = (uint64_t)((saddr >> 4) & 0x3FFFu);
+    d |= (uint64_t)((kBlockBytes >> 4) & 0x3FFF) << 16;
+    d |= (uint64_t)((1024 >> 4) & 0x3FFF) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator,
+// bf16 A and B, both MN-major, N = 256, M = 128.
+constexpr uint32_t kInstrDesc = (1u << 4)               // D: f32
+                                | (1u << 7)             // A: bf16
+                                | (1u << 10)            // B: bf16
+                                | (1u << 15)            // A MN-major
+                                | (1u << 16)            // B MN-major
+                                | ((uint32_t)(kBN >> 3) << 17)
+                                | ((uint32_t)(kBM >> 4) << 24);
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(kInstrDesc), "r"(acc)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+// 32 consecutive fp32 accumulator columns of this thread's lane.
+__device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32])
+{
+    uint32_t r[32];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+        v[e] = __uint_as_float(r[e]);
+}
+
+// Named barrier 1 over the 128 epilogue threads.
+__device__ __forceinline__ void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// Same barrier with an OR over the threads' flags: every epilogue thread gets
+// the same answer, so the four warps always take the same branch.
+__device__ __forceinline__ bool epi_bar_any(bool c)
+{
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "bar.red.or.pred q, 1, 128, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)c)
+        : "memory");
+    return r != 0;
+}
+
+__device__ void set_timeout(volatile int *abort, unsigned *flags)
+{
+    *abort = 1;
+    atomicOr(flags, kFlagTimeout);
+}
+
+// G = dlogits^T H over tiles tile0, tile0 + gridDim.x, ...  Outputs:
+//   G        V x D fp32, row-major
+//   colpart  [ceil(V/128)][D]: sum of g^2 over the 128 rows of each row block
+//   rowpart  [ceil(D/256)][V]: sum of g^2 over the 256 columns of each column block
+__global__ void __launch_bounds__(kLmThreads, 1)
+k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__ CUtensorMap tm_h,
+              float *__restrict__ G, float *__restrict__ colpart, float *__restrict__ rowpart,
+              unsigned *flags, int V, int D, int T)
+{
+    extern __shared__ unsigned char lm_smem_raw[];
+    unsigned char *smem = reinterpret_cast<unsigned char *>(
+        (reinterpret_cast<uintptr_t>(lm_smem_raw) + 1023) & ~(uintptr_t)1023);
+    LmSmemTail *tail = reinterpret_cast<LmSmemTail *>(smem + (size_t)kStages * kStageBytes);
+    volatile int *abort = &tail->abort;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int mblocks = (V + kBM - 1) / kBM;
+    const int nblocks = (D + kBN - 1) / kBN;
+    const int ntiles = mblocks * nblocks;
+    const int kblocks = (T + kBK - 1) / kBK;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(smem_addr(&tail->full[s]), 1);
+            mbar_init(smem_addr(&tail->empty[s]), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(smem_addr(&tail->tfull[a]), 1);
+            mbar_init(smem_addr(&tail->tempty[a]), 4);  // one arrival per epilogue warp
+        }
+        mbar_init(smem_addr(&tail->drain), 1);
+        tail->abort = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_dl)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_h)) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_addr(&tail->tmem_base)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tail->tmem_base;
+    // the state pass may begin launching; it waits for this grid to finish
+    dev::grid_dep_launch();
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t last_parity[kStages];
+        bool issued[kStages];
+        for (int s = 0; s < kStages; ++s) {
+            issued[s] = false;
+            last_parity[s] = 0;
+        }
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+            const int mb = tile / nblocks;
+            const int nb = tile - mb * nblocks;
+            for (int kb = 0; kb < kblocks; ++kb) {
+                if (!mbar_wait(smem_addr(&tail->empty[stage]), phase ^ 1u, abort)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t bar = smem_addr(&tail->full[stage]);
+                mbar_expect_tx(bar, kStageBytes);
+                issued[stage] = true;
+                last_parity[stage] = phase;
+                const uint32_t a_dst = smem_addr(smem + (size_t)stage * kStageBytes);
+                const uint32_t b_dst = a_dst + kABytes;
+                const int y = kb * kBK;
+#pragma unroll
+                for (int j = 0; j < kBM / kBox; ++j)
+                    tma_load_2d(a_dst + j * kBlockBytes, &tm_dl, mb * kBM + j * kBox, y, bar);
+#pragma unroll
+                for (int j = 0; j < kBN / kBox; ++j)
+                    tma_load_2d(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar);
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+        if (!ok)
+            set_timeout(abort, flags);
+        // After an abort elsewhere, copies already issued may still be on
+        // their way into this CTA's shared memory: wait for the last one of
+        // each stage before the CTA may exit (immediate when all were used).
+        for (int s = 0; s < kStages; ++s)
+            if (issued[s])
+                mbar_wait_final(smem_addr(&tail->full[s]), last_parity[s]);
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        int stage = 0;
+        uint32_t phase = 0;
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        bool ok = true;
+        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+            if (!mbar_wait(smem_addr(&tail->tempty[acc]), acc_phase ^ 1u, abort)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t d_tmem = tmem + (uint32_t)(acc * kAccCols);
+            for (int kb = 0; kb < kblocks; ++kb) {
+                if (!mbar_wait(smem_addr(&tail->full[stage]), phase, abort)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t a_base = smem_addr(smem + (size_t)stage * kStageBytes);
+                const uint32_t b_base = a_base + kABytes;
+#pragma unroll
+                for (int k = 0; k < kBK / kUK; ++k) {
+                    // K step k: token rows 16k .. 16k+15 of every box, 2 KiB further on
+                    const uint64_t ad = mn_major_sw128_desc(a_base + (uint32_t)(k * kUK * 128));
+                    const uint64_t bd = mn_major_sw128_desc(b_base + (uint32_t)(k * kUK * 128));
+                    mma_bf16(d_tmem, ad, bd, (kb | k) != 0);
+                }
+                mma_commit(smem_addr(&tail->empty[stage]));
+                if (++stage == kStages) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok)
+                break;
+            mma_commit(smem_addr(&tail->tfull[acc]));
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+        if (!ok)
+            set_timeout(abort, flags);
+        // every MMA issued above completes before the accumulators are freed
+        mma_commit(smem_addr(&tail->drain));
+        mbar_wait_final(smem_addr(&tail->drain), 0);
+    } else if (warp >= kEpiWarp0) {
+        // ---------------- epilogue ----------------
+        const int q = warp - kEpiWarp0;  // accumulator lanes 32q .. 32q+31
+        int acc = 0;
+        uint32_t acc_phase = 0;
+        int buf = 0;
+        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
+            const int mb = tile / nblocks;
+            const int nb = tile - mb * nblocks;
+            bool fail = !mbar_wait(smem_addr(&tail->tfull[acc]), acc_phase, abort);
+            if (fail && !*abort)
+                set_timeout(abort, flags);
+            fail = fail || *abort;
+            if (epi_bar_any(fail))  // all four warps leave together
+                break;
+            tc_fence_after();
+            const int row = mb * kBM + q * 32 + lane;
+            float rowsq = 0.f;
+#pragma unroll 1
+            for (int ch = 0; ch < kBN / 32; ++ch) {
+                float v[32];
+                tmem_load32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kAccCols + ch * 32), v);
+                const int col0 = nb * kBN + ch * 32;
+                if (row < V) {
+                    float *gp = G + (int64_t)row * D + col0;
+                    if (col0 + 32 <= D) {
+#pragma unroll
+                        for (int e = 0; e < 32; e += 4)
+                            *reinterpret_cast<float4 *>(gp + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
+                    } else {
+                        for (int e = 0; e < 32; ++e)
+                            if (col0 + e < D)
+                                gp[e] = v[e];
+                    }
+                }
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    v[e] = v[e] * v[e];
+                    rowsq += v[e];
+                }
+                int col_of_lane;
+                const float cs = dev::warp_sum_transposed<32>(v, lane, col_of_lane);
+                tail->xch[buf][q][col_of_lane] = cs;
+                epi_bar();
+                if (q == 0 && col0 + lane < D)
+                    colpart[(int64_t)mb * D + col0 + lane] =
+                        ((tail->xch[buf][0][lane] + tail->xch[buf][1][lane]) + tail->xch[buf][2][lane]) +
+                        tail->xch[buf][3][lane];
+                buf ^= 1;
+            }
+            if (row < V)
+                rowpart[(int64_t)nb * V + row] = rowsq;
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(smem_addr(&tail->tempty[acc]));
+            if (++acc == 2) {
+                acc = 0;
+                acc_phase ^= 1u;
+            }
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        __syncwarp();
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                     : "memory");
+    }
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
+{
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    });
+    return fn;
+}
+
+// T x n bf16, row-major, loaded as 64 x 64 boxes with the 128-byte swizzle.
+bool make_map(CUtensorMap *m, const void *base, int64_t n, int64_t T)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn)
+        return false;
+    cuuint64_t dims[2] = {(cuuint64_t)n, (cuuint64_t)T};
+    cuuint64_t strides[1] = {(cuuint64_t)n * 2};
+    cuuint32_t box[2] = {(cuuint32_t)kBox, (cuuint32_t)kBK};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+int lmhead_row_blocks(int64_t V) { return (int)((V + kBM - 1) / kBM); }
+int lmhead_col_blocks(int64_t D) { return (int)((D + kBN - 1) / kBN); }
+
+cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
+                               cudaStream_t stream)
+{
+    CUtensorMap tm_dl, tm_h;
+    if (!make_map(&tm_dl, a.dlogits, a.V, a.T) || !make_map(&tm_h, a.hidden, a.D, a.T))
+        return cudaErrorInvalidValue;
+    // per device and cheap: set on every call
+    cudaError_t e = cudaFuncSetAttribute(k_lmhead_grad, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kLmSmemBytes);
+    if (e != cudaSuccess)
+        return e;
+    const int ntiles = lmhead_row_blocks(a.V) * lmhead_col_blocks(a.D);
+    const int grid = ntiles < kSms ? ntiles : kSms;
+    return launch_k(k_lmhead_grad, dim3(grid), dim3(kLmThreads), kLmSmemBytes, stream, false, tm_dl, tm_h,
+                    a.G, colpart, rowpart, flags, (int)a.V, (int)a.D, (int)a.T);
+}
+
+}  // namespace ember

@@ -38,6 +38,7 @@ EXPORTS = (
     "ember_step_sparse", "ember_get_device_status", "ember_status_string",
     "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
     "ember_step_dense_noalloc", "ember_step_dense_from_host",
+    "ember_lmhead_grad", "ember_step_lmhead",
 )
 
 
@@ -84,6 +85,8 @@ def lib():
             "ember_sparse_unique": (st, [vp, vp, ip, i64, vp, vp, vp, vp]),
             "ember_step_dense_noalloc": (st, [vp, vp, vp, vp, flt, i64, vp]),
             "ember_step_dense_from_host": (st, [vp, vp, vp, vp, vp, flt, i64, vp]),
+            "ember_lmhead_grad": (st, [vp, vp, vp, i64, vp, vp]),
+            "ember_step_lmhead": (st, [vp, vp, vp, vp, i64, vp, vp, flt, i64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -171,6 +174,18 @@ def ember_step_dense_from_host(h, W, G_host, G_stage, state, lr, t, stream=None)
                                             lr, t, _stream(stream)), "ember_step_dense_from_host")
 
 
+def ember_lmhead_grad(h, dlogits, hidden, T, G, stream=None):
+    """G = dlogits^T hidden on the tensor cores (dlogits T x V, hidden T x D, bf16)."""
+    _check(lib().ember_lmhead_grad(h, _addr(dlogits), _addr(hidden), T, _addr(G), _stream(stream)),
+           "ember_lmhead_grad")
+
+
+def ember_step_lmhead(h, W, dlogits, hidden, T, G, state, lr, t, stream=None):
+    """The dense step on G = dlogits^T hidden, formed (and written to G) here."""
+    _check(lib().ember_step_lmhead(h, _addr(W), _addr(dlogits), _addr(hidden), T, _addr(G), _addr(state),
+                                   lr, t, _stream(stream)), "ember_step_lmhead")
+
+
 def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
     _check(lib().ember_step_sparse(h, _addr(W), _addr(ids), idtype, N, _addr(rows), _addr(state),
                                    lr, t, _stream(stream)), "ember_step_sparse")
@@ -234,6 +249,14 @@ class Ember:
 
     def step_dense_from_host(self, W, G_host, G_stage, lr, t, stream=None):
         ember_step_dense_from_host(self.handle, W, G_host, G_stage, self.state, lr, t, stream)
+
+    def lmhead_grad(self, dlogits, hidden, G, stream=None):
+        """G (V x D fp32) = dlogits^T hidden; dlogits T x V and hidden T x D bf16."""
+        ember_lmhead_grad(self.handle, dlogits, hidden, dlogits.shape[0], G, stream)
+
+    def step_lmhead(self, W, dlogits, hidden, G, lr, t, stream=None):
+        """One step of an LM head whose gradient dlogits^T hidden is formed into G."""
+        ember_step_lmhead(self.handle, W, dlogits, hidden, dlogits.shape[0], G, self.state, lr, t, stream)
 
     def step_sparse(self, W, ids, rows, lr, t, stream=None):
         import torch

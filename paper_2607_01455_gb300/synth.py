@@ -21,7 +21,14 @@ Alpaca and Countdown; none of that data is used or needed):
 * the sparse workload draws N token ids per step i.i.d. from Zipf(1.1)
   truncated to [0, V) (p_k proportional to (k + 1)^-1.1, inverse CDF in
   fp64 on uniform draws; duplicates kept) and one gradient row per
-  occurrence, i.i.d. N(0, (1e-4)^2).
+  occurrence, i.i.d. N(0, (1e-4)^2);
+* the LM-head gradient workload draws, per step, the two factors of the
+  head's gradient for T tokens (appendix "Decomposing the Squared
+  Gradient"): logits i.i.d. N(0, 2^2) per token, the softmax error
+  dlogits[t] = (softmax(logits_t) - onehot(y_t)) / T with targets y_t
+  i.i.d. Zipf(1.1) as above, and hidden states i.i.d. N(0, 1); both are
+  stored as bfloat16.  G = dlogits^T H then has the Zipf row-energy profile
+  of a trained head (frequent targets carry the largest rows).
 
 Seeds: W_0 uses seed * 1_000_003; step t (t >= 1) uses
 seed * 1_000_003 + t on a generator of the target device; the fixed row sets
@@ -49,6 +56,7 @@ class Workload:
     zero_frac: float = 0.0
     heavy_frac: float = 0.0
     lr: float = 1e-3
+    T: int = 0           # tokens per LM-head gradient
 
 
 WORKLOADS = {
@@ -59,10 +67,14 @@ WORKLOADS = {
         Workload("sparse_v262144_d2048_bf16_n32768", 262144, 2048, "bf16", 100, kind="sparse",
                  N=8 * 4096),
         Workload("dense_lmhead_v128256_d8192_bf16", 128256, 8192, "bf16", 50, heavy_frac=0.01),
+        Workload("lmhead_grad_v128256_d8192_t4096_bf16", 128256, 8192, "bf16", 20, kind="lmhead",
+                 T=4096),
     ]
 }
-# The five workloads in the order they are listed for the paper's method.
-ORDER = list(WORKLOADS)
+# The five workloads of the optimizer step in the order they are listed for
+# the paper's method; the LM-head gradient workload comes after them.
+ORDER = [n for n, w in WORKLOADS.items() if w.kind != "lmhead"]
+LOGIT_STD = 2.0
 
 
 def torch_wdtype(wl):
@@ -138,3 +150,20 @@ def sparse_batch(wl, seed, t, device="cuda", N=None):
     ids = torch.searchsorted(zipf_cdf(wl.V, device), u, right=True).clamp_(max=wl.V - 1)
     rows = torch.randn(N, wl.D, generator=g, device=device, dtype=torch.float32) * SPARSE_STD
     return ids.to(torch.int64), rows
+
+
+def lmhead_inputs(V, D, T, seed, t, device="cuda", chunk=512):
+    """(dlogits bf16 [T, V], hidden bf16 [T, D]) of step t (t >= 1): the
+    softmax error of T tokens, already divided by T, and their hidden states."""
+    g = _gen(device, seed * 1_000_003 + t)
+    u = torch.rand(T, generator=g, device=device, dtype=torch.float64)
+    y = torch.searchsorted(zipf_cdf(V, device), u, right=True).clamp_(max=V - 1)
+    dl = torch.empty(T, V, device=device, dtype=torch.bfloat16)
+    for t0 in range(0, T, chunk):
+        t1 = min(T, t0 + chunk)
+        z = torch.randn(t1 - t0, V, generator=g, device=device, dtype=torch.float32) * LOGIT_STD
+        q = torch.softmax(z, dim=1)
+        q[torch.arange(t1 - t0, device=device), y[t0:t1]] -= 1.0
+        dl[t0:t1] = (q / T).to(torch.bfloat16)
+    hidden = torch.randn(T, D, generator=g, device=device, dtype=torch.float32).to(torch.bfloat16)
+    return dl, hidden

@@ -112,6 +112,18 @@ def test_from_host_refuses_row_only_variant():
         E.ember_destroy(h)
 
 
+@pytest.mark.parametrize("V,D", [(12, 16), (16, 12), (1001, 8)])
+def test_lmhead_needs_multiples_of_8(V, D):
+    h = E.ember_create(V, D)
+    try:
+        fake = 1 << 20
+        assert E.lib().ember_lmhead_grad(h, fake, fake, 4, fake, None) == E.EMBER_ERR_UNSUPPORTED
+        assert E.lib().ember_step_lmhead(h, fake, fake, fake, 4, fake, fake, 1e-3, 1, None) == \
+            E.EMBER_ERR_UNSUPPORTED
+    finally:
+        E.ember_destroy(h)
+
+
 def test_create_accepts_limits():
     for V, D in [(1, 8192), (3, 2048), (2, 2047), (1, 3)]:
         E.ember_destroy(E.ember_create(V, D))
@@ -150,6 +162,18 @@ def test_step_and_bind_reject_on_host():
         assert fh(h, fake, fake, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
         assert fh(h, fake, fake + 2, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_ALIGNMENT
         assert fh(h, fake, fake, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
+        # LM-head gradient and fused step: rejected before any CUDA call
+        lg, sl = lib.ember_lmhead_grad, lib.ember_step_lmhead
+        assert lg(h, None, fake, 4, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert lg(h, fake, fake, 0, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert lg(h, fake, fake, 1 << 31, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert lg(h, fake + 8, fake, 4, fake, None) == E.EMBER_ERR_ALIGNMENT
+        assert lg(h, fake, fake, 4, fake + 4, None) == E.EMBER_ERR_ALIGNMENT
+        assert lg(h, fake, fake, 4, fake, None) == E.EMBER_ERR_WORKSPACE
+        assert sl(h, fake, fake, fake, 4, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
+        assert sl(h, None, fake, fake, 4, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert sl(h, fake, fake, fake, 4, fake, fake, float("inf"), 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert sl(h, fake, fake, fake, 4, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
         assert E.lib().ember_get_device_status(h, None) == E.EMBER_ERR_WORKSPACE
         assert lib.ember_get_device_status(None, None) == E.EMBER_ERR_INVALID_ARG
     finally:
