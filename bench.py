@@ -168,6 +168,105 @@ def run_row_only(wl, dev, steps, warmup, flush, W, G):
             "algorithmic_bytes": B, "params_per_s": wl.V * wl.D / (ms * 1e-3), "gpu_launches": 2 * steps}
 
 
+LMHEAD_KERNELS = ["lmhead_grad", "state", "apply"]
+
+
+def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
+    """The LM-head step fused with the producer of its gradient
+    (ember_step_lmhead: G = dlogits^T H on the tensor cores with the sums of
+    g^2 in the epilogue, then the state and apply passes), against the same
+    step built from cuBLAS (torch.mm, fp32 output) and ember_step_dense."""
+    import torch
+    from paper_2607_01455_gb300 import synth
+    from paper_2607_01455_gb300.ember import Ember
+    V, D, T = wl.V, wl.D, wl.T
+    emb = Ember(V, D, wdtype=wl.wdtype, device=dev)
+    W = synth.init_weights(wl, seed, dev)
+    G = torch.empty(V, D, device=dev)
+    dl, h = synth.lmhead_inputs(V, D, T, seed, 1, dev)
+    nk = len(LMHEAD_KERNELS)
+    t = 0
+    for _ in range(warmup):
+        t += 1
+        flush.zero_()
+        emb.step_lmhead(W, dl, h, G, wl.lr, t)
+    torch.cuda.synchronize()
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(steps)]
+    traced = traced_steps(steps)
+    kern_ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for k in traced}
+    for k in range(steps):
+        t += 1
+        flush.zero_()
+        emb.trace(kern_ev.get(k, []))
+        step_ev[k][0].record()
+        emb.step_lmhead(W, dl, h, G, wl.lr, t)
+        step_ev[k][1].record()
+    torch.cuda.synchronize()
+    emb.trace([])
+    if emb.device_status() != 0:
+        raise SystemExit("device status after the LM-head steps")
+    plain = [k for k in range(steps) if k not in kern_ev]
+    per = {name: sum(kern_ev[k][i].elapsed_time(kern_ev[k][i + 1]) for k in traced) / len(traced)
+           for i, name in enumerate(LMHEAD_KERNELS)}
+    ms = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain)
+
+    # the unfused step: cuBLAS forms G, then the two-pass dense step
+    emb2 = Ember(V, D, wdtype=wl.wdtype, device=dev)
+    dlT = dl.t()
+    try:
+        torch.mm(dlT, h, out_dtype=torch.float32)
+        gemm = lambda: torch.mm(dlT, h, out_dtype=torch.float32)  # noqa: E731
+        cublas_out = "fp32"
+    except (TypeError, RuntimeError):
+        gemm = lambda: torch.mm(dlT, h).float()  # noqa: E731
+        cublas_out = "bf16 then converted"
+    for _ in range(warmup):
+        t += 1
+        flush.zero_()
+        emb2.step_dense(W, gemm(), wl.lr, t)
+    torch.cuda.synchronize()
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
+    for k in range(steps):
+        t += 1
+        flush.zero_()
+        ev[k][0].record()
+        Gc = gemm()
+        ev[k][1].record()
+        emb2.step_dense(W, Gc, wl.lr, t)
+        ev[k][2].record()
+    torch.cuda.synchronize()
+    ms_unfused = sum(e[0].elapsed_time(e[2]) for e in ev) / steps
+    ms_cublas = sum(e[0].elapsed_time(e[1]) for e in ev) / steps
+
+    flops = 2.0 * V * D * T
+    tf = flops / (per["lmhead_grad"] * 1e-3) / 1e12
+    tf_cublas = flops / (ms_cublas * 1e-3) / 1e12
+    peaks = {}
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            pk = json.load(f)
+        peaks = {"burst": float(pk["bf16_tflops"]), "sustained": float(pk["bf16_tflops_sustained"])}
+        peak_kind = "measured"
+    except Exception:
+        peaks = {"burst": 1900.0, "sustained": 1700.0}
+        peak_kind = "fallback"
+    B_fused = (4 + 4 + 2 * wbytes(wl)) * V * D + 2 * T * (V + D)
+    return {"workload": wl.name, "V": V, "D": D, "T": T, "ms_per_step": ms,
+            "kernels_ms": per, "gpu_launches": nk * steps,
+            "roofline": {"bound": "tensor", "kernel": "k_lmhead_grad", "achieved": tf, "peak": peaks["burst"],
+                         "unit": "TFLOP/s", "frac": tf / peaks["burst"],
+                         "frac_of_sustained": tf / peaks["sustained"], "peak_kind": peak_kind,
+                         "flops_per_launch": flops, "traffic": None},
+            "unfused": {"ms_per_step": ms_unfused, "cublas_gemm_ms": ms_cublas, "cublas_tflops": tf_cublas,
+                        "cublas_output": cublas_out,
+                        "what": "torch.mm(dlogits^T, H) then ember_step_dense (reduce, state, apply)"},
+            "speedup_vs_unfused": ms_unfused / ms,
+            "hbm_bytes_fused_step": B_fused,
+            "what": "ember_step_lmhead: G = dlogits^T H (tcgen05, fp32 G written) with per-tile sums of g^2 "
+                    "in the epilogue, state pass, apply pass (G read once)"}
+
+
 def measured_hbm_peak():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -360,6 +459,8 @@ def run_ours(args, world, rank, local):
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     stream = torch.cuda.current_stream(dev)
+    if wl.kind == "lmhead":
+        raise SystemExit("the LM-head gradient workload is timed inside the default line (lmhead_fused)")
     if wl.kind == "sparse":
         return run_sparse_line(args, wl, world, rank, dev)
 
@@ -496,6 +597,12 @@ def run_ours(args, world, rank, local):
         sparse["frac_of_nominal_8TBs"] = sparse["value"] / NOMINAL_HBM_GBS
         sparse["frac_of_measured_hbm"] = sparse["value"] / peak
 
+    lmhead = None
+    if not args.no_lmhead:
+        lwl = synth.WORKLOADS["lmhead_grad_v128256_d8192_t4096_bf16"]
+        lmhead = run_lmhead(lwl, dev, max(2 * TRACE_EVERY, min(args.steps, 20)), args.warmup, flush,
+                            seed=rank)
+
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -517,6 +624,7 @@ def run_ours(args, world, rank, local):
         "wall_s_timed_region": wall,
         "sparse": sparse,
         "row_only": row_only,
+        "lmhead_fused": lmhead,
     }
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -534,6 +642,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-sparse", action="store_true")
     ap.add_argument("--no-row-only", action="store_true")
+    ap.add_argument("--no-lmhead", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

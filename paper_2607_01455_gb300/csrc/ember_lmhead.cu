@@ -15,12 +15,19 @@
 // into the producer of G.
 //
 // Tiles: 128 rows of G (vocabulary) x 256 columns (features), the largest
-// single-CTA tcgen05 shape; 64 tokens per pipeline stage, 4 stages.  Both
-// operands are "MN-major" in memory (dlogits is T x V and H is T x D, row-
-// major, so for fixed token the tile's rows, resp. columns, are contiguous):
-// each stage is loaded by TMA as 64-wide boxes with the 128-byte swizzle and
-// described to the MMA as MN-major, swizzled, 8 KiB between 64-element
-// blocks and 1 KiB between 8-token groups.
+// single-CTA tcgen05 shape; 64 tokens per pipeline stage, 4 stages (192 KiB).
+// Both operands are "MN-major" in memory (dlogits is T x V and H is T x D,
+// row-major, so for a fixed token the tile's rows, resp. columns, are
+// contiguous): each stage is loaded by TMA as 64-wide boxes with the 128-byte
+// swizzle and described to the MMA as MN-major, swizzled, 8 KiB between
+// 64-element blocks and 1 KiB between 8-token groups.
+//
+// Clusters of two CTAs work on two row blocks of the same column block: each
+// loads its own slice of dlogits and half of the slice of H, which TMA
+// multicasts to both, so H costs half the L2 reads.  Tiles are taken in
+// bands of 16 column blocks (all row blocks of a band, then the next band),
+// so the CTAs at work at one time share 32 MiB of H at most; H is loaded
+// with an evict-last L2 policy, dlogits and G stream.
 //
 // Warp roles (256 threads, one CTA per SM, persistent over tiles):
 //   warp 0   one thread issues the TMA loads of every stage
@@ -28,12 +35,14 @@
 //            accumulators, so the epilogue of one tile overlaps the MMAs of
 //            the next); one thread issues the MMAs
 //   warps 4-7  epilogue: warp 4+q reads accumulator lanes 32q..32q+31 (rows
-//            of the tile), stores G, and forms the sums of g^2
+//            of the tile), forms the sums of g^2, and writes each 32 x 32
+//            block of G through swizzled shared memory with a TMA store
+//            (whole 128-byte lines, clipped at the edges of G)
 //
 // Determinism: every output element of G, of the per-tile row sums and of
 // the per-tile column sums is produced by exactly one tile, in a fixed
-// order; nothing is accumulated across CTAs here.  The state pass sums the
-// per-tile partials in a fixed order.
+// order, whatever the grid; nothing is accumulated across CTAs here.  The
+// state pass sums the per-tile partials in a fixed order.
 //
 // Waits on mbarriers are bounded (kWaitNs of wall time); a wait that gives up
 // sets the sticky timeout flag, stops every role, lets the copies and MMAs
@@ -55,7 +64,7 @@ constexpr int kBM = 128;                    // tile rows (UMMA M)
 constexpr int kBN = 256;                    // tile columns (UMMA N)
 constexpr int kBK = 64;                     // tokens per stage
 constexpr int kUK = 16;                     // K of one kind::f16 MMA
-constexpr int kStages = 4;
+constexpr int kStages = 256 / kBK;          // 192 KiB of operand stages
 constexpr int kBox = 64;                    // TMA box: 64 bf16 = 128 bytes, the swizzle span
 constexpr int kABytes = kBM * kBK * 2;      // 16 KiB
 constexpr int kBBytes = kBN * kBK * 2;      // 32 KiB
@@ -66,6 +75,11 @@ constexpr int kTmemCols = 2 * kAccCols;     // two accumulators
 constexpr int kLmThreads = 256;
 constexpr int kEpiWarp0 = 4;
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
+// CTAs per cluster sharing (multicasting) the H slice of one column block.
+// Two: with four, clusters pack the GPCs less well and fewer SMs work.
+constexpr int kLmCluster = 2;
+// Column blocks per band of the tile order (see tile_of).
+constexpr int kLmBand = 16;
 
 // Shared memory: stages (1 KiB aligned for the swizzle), then barriers.
 struct LmSmemTail {
@@ -78,7 +92,12 @@ struct LmSmemTail {
     int abort;
     float xch[2][4][32];       // per-warp column sums, double-buffered
 };
-constexpr size_t kLmSmemBytes = 1024 + (size_t)kStages * kStageBytes + sizeof(LmSmemTail);
+// Epilogue staging of G for the TMA store: per epilogue warp, two 32 x 32
+// fp32 blocks (4 KiB each, 128-byte swizzled rows).
+constexpr int kStoreBlockBytes = 32 * 32 * 4;
+constexpr int kStoreBytes = 4 * 2 * kStoreBlockBytes;
+constexpr size_t kLmSmemBytes = 1024 + (size_t)kStages * kStageBytes + kStoreBytes + sizeof(LmSmemTail);
+static_assert(kLmSmemBytes <= 232448, "over the 227 KiB of shared memory a CTA may use");
 
 __device__ __forceinline__ uint32_t smem_addr(const void *p)
 {
@@ -150,15 +169,46 @@ __device__ bool mbar_wait_final(uint32_t bar, uint32_t parity)
     return true;
 }
 
-__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                            uint32_t bar)
+// L2 eviction policies for the TMA loads (createpolicy; fraction 1.0).
+__device__ __forceinline__ uint64_t l2_policy(int kind)
+{
+    uint64_t p;
+    if (kind == 1)
+        asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    else if (kind == 2)
+        asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    else
+        asm volatile("createpolicy.fractional.L2::evict_normal.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                                 uint32_t bar, uint64_t pol)
 {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol)
         : "memory");
 }
+
+// G block of 32 columns x 32 rows from shared memory to global, clipped at
+// the edges of G by the tensor map; one bulk group per call.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int x, int y, uint64_t pol)
+{
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.bulk_group.L2::cache_hint [%0, {%1, %2}], [%3], %4;" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(x), "r"(y), "r"(src), "l"(pol)
+                 : "memory");
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+}
+// Wait until at most N bulk groups of this thread still read shared memory.
+template <int N>
+__device__ __forceinline__ void tma_store_wait_read()
+{
+    asm volatile("cp.async.bulk.wait_group.read %0;" ::"n"(N) : "memory");
+}
+__device__ __forceinline__ void tma_store_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 
 __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
@@ -248,32 +298,112 @@ __device__ void set_timeout(volatile int *abort, unsigned *flags)
     atomicOr(flags, kFlagTimeout);
 }
 
-// G = dlogits^T H over tiles tile0, tile0 + gridDim.x, ...  Outputs:
-//   G        V x D fp32, row-major
+__device__ __forceinline__ uint32_t cluster_rank()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_id()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%clusterid.x;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_count()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%nclusterid.x;" : "=r"(r));
+    return r;
+}
+// Every thread of every CTA of the cluster: arrive, then wait for all.
+__device__ __forceinline__ void cluster_sync()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+// One 64 x 64 box of H, written to the same shared-memory offset of every
+// CTA in `mask`, each of whose barrier at `bar`'s offset receives the bytes.
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                               uint32_t bar, uint16_t mask, uint64_t pol)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
+        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5, %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask), "l"(pol)
+        : "memory");
+}
+
+// Arrive on the barrier at `bar`'s offset in every CTA of `mask` once the
+// MMAs issued so far by this thread have completed.
+__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask)
+{
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+        "h"(mask)
+        : "memory");
+}
+
+// G = dlogits^T H.  CL CTAs form a cluster that works on CL row blocks of
+// one column block at a time: each CTA loads its own 128 x 64 slice of
+// dlogits per stage and 1/CL of the 64 x 256 slice of H, which TMA
+// multicasts to all CL CTAs, so every byte of H read from L2 feeds CL
+// tiles.  A stage may be refilled once the MMAs of all CL CTAs have read it:
+// each CTA's MMA completion arrives on the "empty" barrier of every CTA in
+// the cluster (count CL).
+// Outputs:
+//   G        V x D fp32, row-major (streaming stores)
 //   colpart  [ceil(V/128)][D]: sum of g^2 over the 128 rows of each row block
 //   rowpart  [ceil(D/256)][V]: sum of g^2 over the 256 columns of each column block
+// Group tile gt -> (row block mb of this CTA, column block nb).  Column
+// blocks are taken in bands of `band`; within a band the row groups go in
+// order and the column blocks of the band vary fastest, so the CTAs working
+// at the same time share few slices of H and few of dlogits.
+__device__ __forceinline__ void tile_of(int gt, int nblocks, int mgroups, int band, int CL, int rank, int &mb,
+                                        int &nb)
+{
+    const int per_band = band * mgroups;
+    const int b = gt / per_band;
+    const int r = gt - b * per_band;
+    const int nb0 = b * band;
+    const int w = (nblocks - nb0 < band) ? nblocks - nb0 : band;  // the last band may be narrower
+    const int mg = r / w;
+    nb = nb0 + (r - mg * w);
+    mb = mg * CL + rank;
+}
+
+template <int CL>
 __global__ void __launch_bounds__(kLmThreads, 1)
 k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__ CUtensorMap tm_h,
-              float *__restrict__ G, float *__restrict__ colpart, float *__restrict__ rowpart,
-              unsigned *flags, int V, int D, int T)
+              const __grid_constant__ CUtensorMap tm_g, float *__restrict__ colpart, float *__restrict__ rowpart,
+              unsigned *flags, int V, int D, int T, int band)
 {
+    static_assert(CL == 1 || CL == 2 || CL == 4, "cluster of 1, 2 or 4 CTAs");
+    constexpr int kBBoxes = kBN / kBox;          // 4 boxes of H per stage
+    constexpr int kMyBoxes = kBBoxes / CL;       // loaded (and multicast) by this CTA
+    constexpr uint16_t kMask = (uint16_t)((1u << CL) - 1u);
     extern __shared__ unsigned char lm_smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(lm_smem_raw) + 1023) & ~(uintptr_t)1023);
-    LmSmemTail *tail = reinterpret_cast<LmSmemTail *>(smem + (size_t)kStages * kStageBytes);
+    unsigned char *gstage = smem + (size_t)kStages * kStageBytes;
+    LmSmemTail *tail = reinterpret_cast<LmSmemTail *>(gstage + kStoreBytes);
     volatile int *abort = &tail->abort;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
     const int mblocks = (V + kBM - 1) / kBM;
     const int nblocks = (D + kBN - 1) / kBN;
-    const int ntiles = mblocks * nblocks;
+    const int mgroups = (mblocks + CL - 1) / CL;
+    const int ngroup_tiles = mgroups * nblocks;
     const int kblocks = (T + kBK - 1) / kBK;
+    const int rank = (CL > 1) ? (int)cluster_rank() : 0;
+    const int gt0 = (CL > 1) ? (int)cluster_id() : (int)blockIdx.x;
+    const int gstep = (CL > 1) ? (int)cluster_count() : (int)gridDim.x;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&tail->full[s]), 1);
-            mbar_init(smem_addr(&tail->empty[s]), 1);
+            mbar_init(smem_addr(&tail->empty[s]), CL);  // the MMAs of every CTA in the cluster
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(smem_addr(&tail->tfull[a]), 1);
@@ -284,6 +414,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_dl)) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_h)) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_g)) : "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -294,6 +425,10 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
     }
     tc_fence_before();
     __syncthreads();
+    // no peer may multicast into this CTA or arrive on its barriers before
+    // they are initialised
+    if constexpr (CL > 1)
+        cluster_sync();
     tc_fence_after();
     const uint32_t tmem = tail->tmem_base;
     // the state pass may begin launching; it waits for this grid to finish
@@ -309,17 +444,20 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
             issued[s] = false;
             last_parity[s] = 0;
         }
+        // H is read by every row group: keep it in L2; dlogits and G stream
+        const uint64_t pol_a = l2_policy(0);
+        const uint64_t pol_b = l2_policy(1);
         bool ok = true;
-        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
-            const int mb = tile / nblocks;
-            const int nb = tile - mb * nblocks;
+        for (int gt = gt0; gt < ngroup_tiles && ok; gt += gstep) {
+            int mb, nb;
+            tile_of(gt, nblocks, mgroups, band, CL, rank, mb, nb);
             for (int kb = 0; kb < kblocks; ++kb) {
                 if (!mbar_wait(smem_addr(&tail->empty[stage]), phase ^ 1u, abort)) {
                     ok = false;
                     break;
                 }
                 const uint32_t bar = smem_addr(&tail->full[stage]);
-                mbar_expect_tx(bar, kStageBytes);
+                mbar_expect_tx(bar, kStageBytes);  // own A + all of the stage's H
                 issued[stage] = true;
                 last_parity[stage] = phase;
                 const uint32_t a_dst = smem_addr(smem + (size_t)stage * kStageBytes);
@@ -327,10 +465,15 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 const int y = kb * kBK;
 #pragma unroll
                 for (int j = 0; j < kBM / kBox; ++j)
-                    tma_load_2d(a_dst + j * kBlockBytes, &tm_dl, mb * kBM + j * kBox, y, bar);
+                    tma_load_2d_hint(a_dst + j * kBlockBytes, &tm_dl, mb * kBM + j * kBox, y, bar, pol_a);
 #pragma unroll
-                for (int j = 0; j < kBN / kBox; ++j)
-                    tma_load_2d(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar);
+                for (int q = 0; q < kMyBoxes; ++q) {
+                    const int j = rank * kMyBoxes + q;
+                    if constexpr (CL > 1)
+                        tma_load_2d_mc(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar, kMask, pol_b);
+                    else
+                        tma_load_2d_hint(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar, pol_b);
+                }
                 if (++stage == kStages) {
                     stage = 0;
                     phase ^= 1u;
@@ -339,9 +482,10 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         }
         if (!ok)
             set_timeout(abort, flags);
-        // After an abort elsewhere, copies already issued may still be on
-        // their way into this CTA's shared memory: wait for the last one of
-        // each stage before the CTA may exit (immediate when all were used).
+        // After an abort, copies already issued (here or by a peer) may still
+        // be on their way into this CTA's shared memory: wait for the last
+        // one of each stage before the CTA may exit (immediate when all were
+        // used; bounded when a peer stopped early).
         for (int s = 0; s < kStages; ++s)
             if (issued[s])
                 mbar_wait_final(smem_addr(&tail->full[s]), last_parity[s]);
@@ -352,7 +496,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         int acc = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int tile = blockIdx.x; tile < ntiles && ok; tile += gridDim.x) {
+        for (int gt = gt0; gt < ngroup_tiles && ok; gt += gstep) {
             if (!mbar_wait(smem_addr(&tail->tempty[acc]), acc_phase ^ 1u, abort)) {
                 ok = false;
                 break;
@@ -374,7 +518,10 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                     const uint64_t bd = mn_major_sw128_desc(b_base + (uint32_t)(k * kUK * 128));
                     mma_bf16(d_tmem, ad, bd, (kb | k) != 0);
                 }
-                mma_commit(smem_addr(&tail->empty[stage]));
+                if constexpr (CL > 1)
+                    mma_commit_mc(smem_addr(&tail->empty[stage]), kMask);
+                else
+                    mma_commit(smem_addr(&tail->empty[stage]));
                 if (++stage == kStages) {
                     stage = 0;
                     phase ^= 1u;
@@ -399,9 +546,12 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         int acc = 0;
         uint32_t acc_phase = 0;
         int buf = 0;
-        for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x) {
-            const int mb = tile / nblocks;
-            const int nb = tile - mb * nblocks;
+        int sbuf = 0;  // which of this warp's two staging blocks
+        unsigned char *my_stage = gstage + (size_t)q * 2 * kStoreBlockBytes;
+        const uint64_t pol_g = l2_policy(2);
+        for (int gt = gt0; gt < ngroup_tiles; gt += gstep) {
+            int mb, nb;
+            tile_of(gt, nblocks, mgroups, band, CL, rank, mb, nb);
             bool fail = !mbar_wait(smem_addr(&tail->tfull[acc]), acc_phase, abort);
             if (fail && !*abort)
                 set_timeout(abort, flags);
@@ -416,17 +566,24 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 float v[32];
                 tmem_load32(tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kAccCols + ch * 32), v);
                 const int col0 = nb * kBN + ch * 32;
-                if (row < V) {
-                    float *gp = G + (int64_t)row * D + col0;
-                    if (col0 + 32 <= D) {
+                const int row0 = mb * kBM + q * 32;
+                // G block (32 rows x 32 columns) through shared memory: row
+                // `lane` is 128 bytes, its 16-byte pieces in the 128-byte
+                // swizzle order; then one TMA store, clipped at V and D
+                if (row0 < V) {
+                    if (lane == 0)
+                        tma_store_wait_read<1>();  // this staging block's previous store has read it
+                    __syncwarp();
+                    unsigned char *blk = my_stage + sbuf * kStoreBlockBytes + lane * 128;
 #pragma unroll
-                        for (int e = 0; e < 32; e += 4)
-                            *reinterpret_cast<float4 *>(gp + e) = make_float4(v[e], v[e + 1], v[e + 2], v[e + 3]);
-                    } else {
-                        for (int e = 0; e < 32; ++e)
-                            if (col0 + e < D)
-                                gp[e] = v[e];
-                    }
+                    for (int c = 0; c < 8; ++c)
+                        *reinterpret_cast<float4 *>(blk + ((c ^ (lane & 7)) << 4)) =
+                            make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    __syncwarp();
+                    if (lane == 0)
+                        tma_store_2d(&tm_g, smem_addr(my_stage + sbuf * kStoreBlockBytes), col0, row0, pol_g);
+                    sbuf ^= 1;
                 }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
@@ -437,7 +594,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 const float cs = dev::warp_sum_transposed<32>(v, lane, col_of_lane);
                 tail->xch[buf][q][col_of_lane] = cs;
                 epi_bar();
-                if (q == 0 && col0 + lane < D)
+                if (q == 0 && mb < mblocks && col0 + lane < D)
                     colpart[(int64_t)mb * D + col0 + lane] =
                         ((tail->xch[buf][0][lane] + tail->xch[buf][1][lane]) + tail->xch[buf][2][lane]) +
                         tail->xch[buf][3][lane];
@@ -456,8 +613,14 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         }
     }
 
+    if (warp >= kEpiWarp0 && lane == 0)
+        tma_store_wait_all();  // the stores of G have completed
     tc_fence_before();
     __syncthreads();
+    // no CTA of the cluster exits while a peer's MMA completion may still
+    // arrive on its barriers
+    if constexpr (CL > 1)
+        cluster_sync();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
@@ -481,6 +644,21 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
+// G, V x D fp32 row-major, stored as 32 x 32 boxes with the 128-byte swizzle.
+bool make_store_map(CUtensorMap *m, float *G, int64_t V, int64_t D)
+{
+    PFN_cuTensorMapEncodeTiled_v12000 fn = encode_fn();
+    if (!fn)
+        return false;
+    cuuint64_t dims[2] = {(cuuint64_t)D, (cuuint64_t)V};
+    cuuint64_t strides[1] = {(cuuint64_t)D * 4};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, G, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+              CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // T x n bf16, row-major, loaded as 64 x 64 boxes with the 128-byte swizzle.
 bool make_map(CUtensorMap *m, const void *base, int64_t n, int64_t T)
 {
@@ -501,21 +679,55 @@ bool make_map(CUtensorMap *m, const void *base, int64_t n, int64_t T)
 int lmhead_row_blocks(int64_t V) { return (int)((V + kBM - 1) / kBM); }
 int lmhead_col_blocks(int64_t D) { return (int)((D + kBN - 1) / kBN); }
 
-cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
-                               cudaStream_t stream)
+namespace {
+
+template <int CL>
+cudaError_t launch_cl(const CUtensorMap &tm_dl, const CUtensorMap &tm_h, const CUtensorMap &tm_g, const LmArgs &a,
+                      float *colpart, float *rowpart, unsigned *flags, cudaStream_t stream)
 {
-    CUtensorMap tm_dl, tm_h;
-    if (!make_map(&tm_dl, a.dlogits, a.V, a.T) || !make_map(&tm_h, a.hidden, a.D, a.T))
-        return cudaErrorInvalidValue;
     // per device and cheap: set on every call
-    cudaError_t e = cudaFuncSetAttribute(k_lmhead_grad, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_lmhead_grad<CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kLmSmemBytes);
     if (e != cudaSuccess)
         return e;
-    const int ntiles = lmhead_row_blocks(a.V) * lmhead_col_blocks(a.D);
-    const int grid = ntiles < kSms ? ntiles : kSms;
-    return launch_k(k_lmhead_grad, dim3(grid), dim3(kLmThreads), kLmSmemBytes, stream, false, tm_dl, tm_h,
-                    a.G, colpart, rowpart, flags, (int)a.V, (int)a.D, (int)a.T);
+    cudaLaunchConfig_t cfg = {};
+    cfg.blockDim = dim3(kLmThreads);
+    cfg.dynamicSmemBytes = kLmSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    // persistent: as many clusters as fit on the GPU at once (clusters are
+    // placed within one GPC, so this can be below kSms / CL)
+    cfg.gridDim = dim3(kSms);
+    int fit = 0;
+    e = cudaOccupancyMaxActiveClusters(&fit, k_lmhead_grad<CL>, &cfg);
+    if (e != cudaSuccess)
+        return e;
+    if (fit < 1)
+        return cudaErrorInvalidConfiguration;
+    const int groups = (lmhead_row_blocks(a.V) + CL - 1) / CL * lmhead_col_blocks(a.D);
+    const int nclusters = groups < fit ? groups : fit;
+    cfg.gridDim = dim3(nclusters * CL);
+    const int band = kLmBand < lmhead_col_blocks(a.D) ? kLmBand : lmhead_col_blocks(a.D);
+    return cudaLaunchKernelEx(&cfg, k_lmhead_grad<CL>, tm_dl, tm_h, tm_g, colpart, rowpart, flags, (int)a.V,
+                              (int)a.D, (int)a.T, band);
+}
+
+}  // namespace
+
+cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
+                               cudaStream_t stream)
+{
+    CUtensorMap tm_dl, tm_h, tm_g;
+    if (!make_map(&tm_dl, a.dlogits, a.V, a.T) || !make_map(&tm_h, a.hidden, a.D, a.T) ||
+        !make_store_map(&tm_g, a.G, a.V, a.D))
+        return cudaErrorInvalidValue;
+    return launch_cl<kLmCluster>(tm_dl, tm_h, tm_g, a, colpart, rowpart, flags, stream);
 }
 
 }  // namespace ember
