@@ -649,9 +649,11 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             return e;
         if (a.trace)
             cudaEventRecord(a.trace[1], a.stream);
+        // plain stream order after the tensor-core kernel: launched early,
+        // the state grid made the step slower (measured 0.1-0.3 ms)
         const int nrow_ctas = kSms;
         e = launch_state(lm_col, lmhead_row_blocks(a.V), rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D,
-                         a.beta2, a.one_minus_beta2, a.inv_bc, a.stream, pdl, a.r, nullptr, lm_row,
+                         a.beta2, a.one_minus_beta2, a.inv_bc, a.stream, false, a.r, nullptr, lm_row,
                          lmhead_col_blocks(a.D), nrow_ctas);
         if (e != cudaSuccess)
             return e;

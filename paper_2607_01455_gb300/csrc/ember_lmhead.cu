@@ -14,26 +14,31 @@
 // and apply passes: the fused deterministic reduction of Section 2.3, moved
 // into the producer of G.
 //
-// Tiles: 128 rows of G (vocabulary) x 256 columns (features), the largest
-// single-CTA tcgen05 shape; 64 tokens per pipeline stage, 4 stages (192 KiB).
+// Tiles: a pair of CTAs (a cluster of two, on two SMs) runs
+// tcgen05.mma.cta_group::2 on 256 rows of G (vocabulary) x 256 columns
+// (features).  Each CTA holds, per pipeline stage of 64 tokens, its own 128
+// rows of dlogits and its own 128 columns of H (32 KiB; six stages, 192 KiB),
+// and its tensor memory holds its 128 rows of the 256 x 256 accumulator; the
+// even CTA (the leader) issues the MMAs for both.  Halving the H each SM
+// stages (the two tensor cores share the halves) is what lets six stages of
+// operands fit, enough to cover L2 latency.
+//
 // Both operands are "MN-major" in memory (dlogits is T x V and H is T x D,
 // row-major, so for a fixed token the tile's rows, resp. columns, are
-// contiguous): each stage is loaded by TMA as 64-wide boxes with the 128-byte
-// swizzle and described to the MMA as MN-major, swizzled, 8 KiB between
-// 64-element blocks and 1 KiB between 8-token groups.
+// contiguous): TMA loads 64 x 64 boxes with the 128-byte swizzle, described to
+// the MMA as MN-major, swizzled, 8 KiB between 64-element blocks and 1 KiB
+// between 8-token groups.  Both CTAs' loads of a stage complete on the
+// leader's barrier; the leader's MMA completion frees the stage in both.
 //
-// Clusters of two CTAs work on two row blocks of the same column block: each
-// loads its own slice of dlogits and half of the slice of H, which TMA
-// multicasts to both, so H costs half the L2 reads.  Tiles are taken in
-// bands of 16 column blocks (all row blocks of a band, then the next band),
-// so the CTAs at work at one time share 32 MiB of H at most; H is loaded
-// with an evict-last L2 policy, dlogits and G stream.
+// Tiles are taken in bands of 16 column blocks (all row pairs of a band, then
+// the next band), so the CTAs at work at one time share 32 MiB of H at most;
+// H is loaded with an evict-last L2 policy, dlogits and G stream.
 //
-// Warp roles (256 threads, one CTA per SM, persistent over tiles):
-//   warp 0   one thread issues the TMA loads of every stage
-//   warp 1   allocates 512 tensor-memory columns (two 128 x 256 fp32
+// Warp roles (256 threads per CTA, one CTA per SM, persistent over tiles):
+//   warp 0   one thread issues the TMA loads of this CTA's halves
+//   warp 1   allocates, with its peer, 512 tensor-memory columns (two
 //            accumulators, so the epilogue of one tile overlaps the MMAs of
-//            the next); one thread issues the MMAs
+//            the next); in the leader one thread issues the MMAs
 //   warps 4-7  epilogue: warp 4+q reads accumulator lanes 32q..32q+31 (rows
 //            of the tile), forms the sums of g^2, and writes each 32 x 32
 //            block of G through swizzled shared memory with a TMA store
@@ -60,14 +65,15 @@
 namespace ember {
 namespace {
 
-constexpr int kBM = 128;                    // tile rows (UMMA M)
+constexpr int kBM = 128;                    // accumulator rows per CTA (half the pair's UMMA M)
+constexpr int kPairM = 2 * kBM;             // UMMA M of the pair
 constexpr int kBN = 256;                    // tile columns (UMMA N)
 constexpr int kBK = 64;                     // tokens per stage
 constexpr int kUK = 16;                     // K of one kind::f16 MMA
-constexpr int kStages = 256 / kBK;          // 192 KiB of operand stages
+constexpr int kStages = 6;
 constexpr int kBox = 64;                    // TMA box: 64 bf16 = 128 bytes, the swizzle span
-constexpr int kABytes = kBM * kBK * 2;      // 16 KiB
-constexpr int kBBytes = kBN * kBK * 2;      // 32 KiB
+constexpr int kABytes = kBM * kBK * 2;      // 16 KiB: this CTA's 128 rows of dlogits
+constexpr int kBBytes = (kBN / 2) * kBK * 2;  // 16 KiB: this CTA's 128 columns of H
 constexpr int kStageBytes = kABytes + kBBytes;
 constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 8 KiB
 constexpr int kAccCols = kBN;               // fp32 accumulator columns per tile
@@ -75,19 +81,16 @@ constexpr int kTmemCols = 2 * kAccCols;     // two accumulators
 constexpr int kLmThreads = 256;
 constexpr int kEpiWarp0 = 4;
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s
-// CTAs per cluster sharing (multicasting) the H slice of one column block.
-// Two: with four, clusters pack the GPCs less well and fewer SMs work.
-constexpr int kLmCluster = 2;
 // Column blocks per band of the tile order (see tile_of).
 constexpr int kLmBand = 16;
 
-// Shared memory: stages (1 KiB aligned for the swizzle), then barriers.
+// Shared memory: stages (1 KiB aligned for the swizzle), G staging, barriers.
 struct LmSmemTail {
-    uint64_t full[kStages];    // TMA bytes landed
-    uint64_t empty[kStages];   // MMAs of the stage done
-    uint64_t tfull[2];         // accumulator ready for the epilogue
-    uint64_t tempty[2];        // accumulator drained by the epilogue
-    uint64_t drain;            // every MMA issued has completed
+    uint64_t full[kStages];    // leader: both CTAs' bytes of the stage landed
+    uint64_t empty[kStages];   // each CTA: the pair's MMAs of the stage done
+    uint64_t tfull[2];         // each CTA: accumulator ready for the epilogue
+    uint64_t tempty[2];        // leader: both CTAs' epilogues drained the accumulator
+    uint64_t drain;            // leader: every MMA issued has completed
     uint32_t tmem_base;
     int abort;
     float xch[2][4][32];       // per-warp column sums, double-buffered
@@ -120,11 +123,6 @@ __device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes)
 {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
                  : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
@@ -182,16 +180,6 @@ __device__ __forceinline__ uint64_t l2_policy(int kind)
     return p;
 }
 
-__device__ __forceinline__ void tma_load_2d_hint(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                                 uint32_t bar, uint64_t pol)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
-        " [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol)
-        : "memory");
-}
-
 // G block of 32 columns x 32 rows from shared memory to global, clipped at
 // the edges of G by the tensor map; one bulk group per call.
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int x, int y, uint64_t pol)
@@ -228,30 +216,14 @@ __device__ __forceinline__ uint64_t mn_major_sw128_desc(uint32_t saddr)
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator,
-// bf16 A and B, both MN-major, N = 256, M = 128.
+// bf16 A and B, both MN-major, N = 256, M = 256 (the pair).
 constexpr uint32_t kInstrDesc = (1u << 4)               // D: f32
                                 | (1u << 7)             // A: bf16
                                 | (1u << 10)            // B: bf16
                                 | (1u << 15)            // A MN-major
                                 | (1u << 16)            // B MN-major
                                 | ((uint32_t)(kBN >> 3) << 17)
-                                | ((uint32_t)(kBM >> 4) << 24);
-
-__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(a), "l"(b), "r"(kInstrDesc), "r"(acc)
-        : "memory");
-}
-
-__device__ __forceinline__ void mma_commit(uint32_t bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
-}
+                                | ((uint32_t)(kPairM >> 4) << 24);
 
 // 32 consecutive fp32 accumulator columns of this thread's lane.
 __device__ __forceinline__ void tmem_load32(uint32_t taddr, float (&v)[32])
@@ -322,66 +294,82 @@ __device__ __forceinline__ void cluster_sync()
     asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-// One 64 x 64 box of H, written to the same shared-memory offset of every
-// CTA in `mask`, each of whose barrier at `bar`'s offset receives the bytes.
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, int x, int y,
-                                               uint32_t bar, uint16_t mask, uint64_t pol)
+// Address of the same shared-memory variable in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t mapa_rank(uint32_t addr, uint32_t rank)
+{
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr)
+{
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+// One 64 x 64 box into this CTA's shared memory; its bytes complete on the
+// barrier `bar` (a cluster address: the leader's barrier for both CTAs).
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y, uint32_t bar,
+                                            uint64_t pol)
 {
     asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5, %6;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "h"(mask), "l"(pol)
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.cta_group::2"
+        ".L2::cache_hint [%0], [%1, {%2, %3}], [%4], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar), "l"(pol)
         : "memory");
 }
 
-// Arrive on the barrier at `bar`'s offset in every CTA of `mask` once the
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t acc)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(kInstrDesc), "r"(acc)
+        : "memory");
+}
+
+// Arrive on the barrier at `bar`'s offset in both CTAs of the pair once the
 // MMAs issued so far by this thread have completed.
-__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask)
+__device__ __forceinline__ void mma_commit_mc(uint32_t bar)
 {
     asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
-        "h"(mask)
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+        "h"((uint16_t)3)
         : "memory");
 }
 
-// G = dlogits^T H.  CL CTAs form a cluster that works on CL row blocks of
-// one column block at a time: each CTA loads its own 128 x 64 slice of
-// dlogits per stage and 1/CL of the 64 x 256 slice of H, which TMA
-// multicasts to all CL CTAs, so every byte of H read from L2 feeds CL
-// tiles.  A stage may be refilled once the MMAs of all CL CTAs have read it:
-// each CTA's MMA completion arrives on the "empty" barrier of every CTA in
-// the cluster (count CL).
-// Outputs:
-//   G        V x D fp32, row-major (streaming stores)
-//   colpart  [ceil(V/128)][D]: sum of g^2 over the 128 rows of each row block
-//   rowpart  [ceil(D/256)][V]: sum of g^2 over the 256 columns of each column block
-// Group tile gt -> (row block mb of this CTA, column block nb).  Column
-// blocks are taken in bands of `band`; within a band the row groups go in
+__device__ __forceinline__ void mma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+// Pair tile gt -> (row block mb of this CTA, column block nb).  Column
+// blocks are taken in bands of `band`; within a band the row pairs go in
 // order and the column blocks of the band vary fastest, so the CTAs working
 // at the same time share few slices of H and few of dlogits.
-__device__ __forceinline__ void tile_of(int gt, int nblocks, int mgroups, int band, int CL, int rank, int &mb,
-                                        int &nb)
+__device__ __forceinline__ void tile_of(int gt, int nblocks, int mpairs, int band, int rank, int &mb, int &nb)
 {
-    const int per_band = band * mgroups;
+    const int per_band = band * mpairs;
     const int b = gt / per_band;
     const int r = gt - b * per_band;
     const int nb0 = b * band;
     const int w = (nblocks - nb0 < band) ? nblocks - nb0 : band;  // the last band may be narrower
-    const int mg = r / w;
-    nb = nb0 + (r - mg * w);
-    mb = mg * CL + rank;
+    const int mp = r / w;
+    nb = nb0 + (r - mp * w);
+    mb = mp * 2 + rank;
 }
 
-template <int CL>
+// G = dlogits^T H, one CTA of a pair.  Outputs:
+//   G        V x D fp32, row-major (TMA stores through tm_g)
+//   colpart  [ceil(V/128)][D]: sum of g^2 over the 128 rows of each row block
+//   rowpart  [ceil(D/256)][V]: sum of g^2 over the 256 columns of each column block
 __global__ void __launch_bounds__(kLmThreads, 1)
 k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__ CUtensorMap tm_h,
               const __grid_constant__ CUtensorMap tm_g, float *__restrict__ colpart, float *__restrict__ rowpart,
               unsigned *flags, int V, int D, int T, int band)
 {
-    static_assert(CL == 1 || CL == 2 || CL == 4, "cluster of 1, 2 or 4 CTAs");
-    constexpr int kBBoxes = kBN / kBox;          // 4 boxes of H per stage
-    constexpr int kMyBoxes = kBBoxes / CL;       // loaded (and multicast) by this CTA
-    constexpr uint16_t kMask = (uint16_t)((1u << CL) - 1u);
     extern __shared__ unsigned char lm_smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
         (reinterpret_cast<uintptr_t>(lm_smem_raw) + 1023) & ~(uintptr_t)1023);
@@ -393,21 +381,22 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
     const int lane = threadIdx.x & 31;
     const int mblocks = (V + kBM - 1) / kBM;
     const int nblocks = (D + kBN - 1) / kBN;
-    const int mgroups = (mblocks + CL - 1) / CL;
-    const int ngroup_tiles = mgroups * nblocks;
+    const int mpairs = (mblocks + 1) / 2;
+    const int npair_tiles = mpairs * nblocks;
     const int kblocks = (T + kBK - 1) / kBK;
-    const int rank = (CL > 1) ? (int)cluster_rank() : 0;
-    const int gt0 = (CL > 1) ? (int)cluster_id() : (int)blockIdx.x;
-    const int gstep = (CL > 1) ? (int)cluster_count() : (int)gridDim.x;
+    const int rank = (int)cluster_rank();
+    const bool leader = rank == 0;
+    const int gt0 = (int)cluster_id();
+    const int gstep = (int)cluster_count();
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < kStages; ++s) {
             mbar_init(smem_addr(&tail->full[s]), 1);
-            mbar_init(smem_addr(&tail->empty[s]), CL);  // the MMAs of every CTA in the cluster
+            mbar_init(smem_addr(&tail->empty[s]), 1);
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(smem_addr(&tail->tfull[a]), 1);
-            mbar_init(smem_addr(&tail->tempty[a]), 4);  // one arrival per epilogue warp
+            mbar_init(smem_addr(&tail->tempty[a]), 8);  // four epilogue warps in each CTA
         }
         mbar_init(smem_addr(&tail->drain), 1);
         tail->abort = 0;
@@ -417,25 +406,22 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&tm_g)) : "memory");
     }
     if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+        // one warp in each CTA of the pair allocates, together
+        asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_addr(&tail->tmem_base)),
                      "r"(kTmemCols)
                      : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
     }
     tc_fence_before();
     __syncthreads();
-    // no peer may multicast into this CTA or arrive on its barriers before
-    // they are initialised
-    if constexpr (CL > 1)
-        cluster_sync();
+    // no peer may signal this CTA's barriers before they are initialised
+    cluster_sync();
     tc_fence_after();
     const uint32_t tmem = tail->tmem_base;
-    // the state pass may begin launching; it waits for this grid to finish
-    dev::grid_dep_launch();
 
     if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer ----------------
+        // ---------------- TMA producer (both CTAs) ----------------
         int stage = 0;
         uint32_t phase = 0;
         uint32_t last_parity[kStages];
@@ -444,20 +430,22 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
             issued[s] = false;
             last_parity[s] = 0;
         }
-        // H is read by every row group: keep it in L2; dlogits and G stream
         const uint64_t pol_a = l2_policy(0);
         const uint64_t pol_b = l2_policy(1);
         bool ok = true;
-        for (int gt = gt0; gt < ngroup_tiles && ok; gt += gstep) {
+        for (int gt = gt0; gt < npair_tiles && ok; gt += gstep) {
             int mb, nb;
-            tile_of(gt, nblocks, mgroups, band, CL, rank, mb, nb);
+            tile_of(gt, nblocks, mpairs, band, rank, mb, nb);
             for (int kb = 0; kb < kblocks; ++kb) {
+                // both CTAs' halves of this stage were read by the pair's MMAs
                 if (!mbar_wait(smem_addr(&tail->empty[stage]), phase ^ 1u, abort)) {
                     ok = false;
                     break;
                 }
-                const uint32_t bar = smem_addr(&tail->full[stage]);
-                mbar_expect_tx(bar, kStageBytes);  // own A + all of the stage's H
+                const uint32_t my_full = smem_addr(&tail->full[stage]);
+                if (leader)
+                    mbar_expect_tx(my_full, 2 * kStageBytes);  // both CTAs' bytes land on the leader's barrier
+                const uint32_t bar = mapa_rank(my_full, 0);
                 issued[stage] = true;
                 last_parity[stage] = phase;
                 const uint32_t a_dst = smem_addr(smem + (size_t)stage * kStageBytes);
@@ -465,15 +453,11 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 const int y = kb * kBK;
 #pragma unroll
                 for (int j = 0; j < kBM / kBox; ++j)
-                    tma_load_2d_hint(a_dst + j * kBlockBytes, &tm_dl, mb * kBM + j * kBox, y, bar, pol_a);
+                    tma_load_2d(a_dst + j * kBlockBytes, &tm_dl, mb * kBM + j * kBox, y, bar, pol_a);
 #pragma unroll
-                for (int q = 0; q < kMyBoxes; ++q) {
-                    const int j = rank * kMyBoxes + q;
-                    if constexpr (CL > 1)
-                        tma_load_2d_mc(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar, kMask, pol_b);
-                    else
-                        tma_load_2d_hint(b_dst + j * kBlockBytes, &tm_h, nb * kBN + j * kBox, y, bar, pol_b);
-                }
+                for (int j = 0; j < (kBN / 2) / kBox; ++j)
+                    tma_load_2d(b_dst + j * kBlockBytes, &tm_h, nb * kBN + rank * (kBN / 2) + j * kBox, y,
+                                bar, pol_b);
                 if (++stage == kStages) {
                     stage = 0;
                     phase ^= 1u;
@@ -482,21 +466,22 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         }
         if (!ok)
             set_timeout(abort, flags);
-        // After an abort, copies already issued (here or by a peer) may still
-        // be on their way into this CTA's shared memory: wait for the last
-        // one of each stage before the CTA may exit (immediate when all were
-        // used; bounded when a peer stopped early).
-        for (int s = 0; s < kStages; ++s)
-            if (issued[s])
-                mbar_wait_final(smem_addr(&tail->full[s]), last_parity[s]);
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer ----------------
+        // After an abort, copies already issued may still be on their way:
+        // the leader waits for the last phase of each stage (both CTAs'
+        // bytes complete there; immediate when every stage was consumed)
+        // before the pair meets at the final cluster barrier.
+        if (leader)
+            for (int s = 0; s < kStages; ++s)
+                if (issued[s])
+                    mbar_wait_final(smem_addr(&tail->full[s]), last_parity[s]);
+    } else if (warp == 1 && lane == 0 && leader) {
+        // ---------------- MMA issuer (leader only) ----------------
         int stage = 0;
         uint32_t phase = 0;
         int acc = 0;
         uint32_t acc_phase = 0;
         bool ok = true;
-        for (int gt = gt0; gt < ngroup_tiles && ok; gt += gstep) {
+        for (int gt = gt0; gt < npair_tiles && ok; gt += gstep) {
             if (!mbar_wait(smem_addr(&tail->tempty[acc]), acc_phase ^ 1u, abort)) {
                 ok = false;
                 break;
@@ -513,15 +498,13 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 const uint32_t b_base = a_base + kABytes;
 #pragma unroll
                 for (int k = 0; k < kBK / kUK; ++k) {
-                    // K step k: token rows 16k .. 16k+15 of every box, 2 KiB further on
+                    // K step k: token rows 16k .. 16k+15 of every box, 2 KiB further on;
+                    // the same offsets address the peer's halves
                     const uint64_t ad = mn_major_sw128_desc(a_base + (uint32_t)(k * kUK * 128));
                     const uint64_t bd = mn_major_sw128_desc(b_base + (uint32_t)(k * kUK * 128));
                     mma_bf16(d_tmem, ad, bd, (kb | k) != 0);
                 }
-                if constexpr (CL > 1)
-                    mma_commit_mc(smem_addr(&tail->empty[stage]), kMask);
-                else
-                    mma_commit(smem_addr(&tail->empty[stage]));
+                mma_commit_mc(smem_addr(&tail->empty[stage]));
                 if (++stage == kStages) {
                     stage = 0;
                     phase ^= 1u;
@@ -529,7 +512,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
             }
             if (!ok)
                 break;
-            mma_commit(smem_addr(&tail->tfull[acc]));
+            mma_commit_mc(smem_addr(&tail->tfull[acc]));
             if (++acc == 2) {
                 acc = 0;
                 acc_phase ^= 1u;
@@ -537,21 +520,21 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         }
         if (!ok)
             set_timeout(abort, flags);
-        // every MMA issued above completes before the accumulators are freed
+        // every MMA issued above completes before either CTA frees its tensor memory
         mma_commit(smem_addr(&tail->drain));
         mbar_wait_final(smem_addr(&tail->drain), 0);
     } else if (warp >= kEpiWarp0) {
-        // ---------------- epilogue ----------------
+        // ---------------- epilogue (both CTAs) ----------------
         const int q = warp - kEpiWarp0;  // accumulator lanes 32q .. 32q+31
         int acc = 0;
         uint32_t acc_phase = 0;
         int buf = 0;
-        int sbuf = 0;  // which of this warp's two staging blocks
+        int sbuf = 0;
         unsigned char *my_stage = gstage + (size_t)q * 2 * kStoreBlockBytes;
         const uint64_t pol_g = l2_policy(2);
-        for (int gt = gt0; gt < ngroup_tiles; gt += gstep) {
+        for (int gt = gt0; gt < npair_tiles; gt += gstep) {
             int mb, nb;
-            tile_of(gt, nblocks, mgroups, band, CL, rank, mb, nb);
+            tile_of(gt, nblocks, mpairs, band, rank, mb, nb);
             bool fail = !mbar_wait(smem_addr(&tail->tfull[acc]), acc_phase, abort);
             if (fail && !*abort)
                 set_timeout(abort, flags);
@@ -605,7 +588,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
-                mbar_arrive(smem_addr(&tail->tempty[acc]));
+                mbar_arrive_cluster(mapa_rank(smem_addr(&tail->tempty[acc]), 0));  // the leader's barrier
             if (++acc == 2) {
                 acc = 0;
                 acc_phase ^= 1u;
@@ -617,14 +600,13 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         tma_store_wait_all();  // the stores of G have completed
     tc_fence_before();
     __syncthreads();
-    // no CTA of the cluster exits while a peer's MMA completion may still
-    // arrive on its barriers
-    if constexpr (CL > 1)
-        cluster_sync();
+    // neither CTA frees its tensor memory or exits while its peer may still
+    // use them (the leader's MMAs write both; arrivals cross the pair)
+    cluster_sync();
     if (warp == 1) {
         __syncwarp();
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+        asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
                      : "memory");
     }
 }
@@ -679,14 +661,15 @@ bool make_map(CUtensorMap *m, const void *base, int64_t n, int64_t T)
 int lmhead_row_blocks(int64_t V) { return (int)((V + kBM - 1) / kBM); }
 int lmhead_col_blocks(int64_t D) { return (int)((D + kBN - 1) / kBN); }
 
-namespace {
-
-template <int CL>
-cudaError_t launch_cl(const CUtensorMap &tm_dl, const CUtensorMap &tm_h, const CUtensorMap &tm_g, const LmArgs &a,
-                      float *colpart, float *rowpart, unsigned *flags, cudaStream_t stream)
+cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
+                               cudaStream_t stream)
 {
+    CUtensorMap tm_dl, tm_h, tm_g;
+    if (!make_map(&tm_dl, a.dlogits, a.V, a.T) || !make_map(&tm_h, a.hidden, a.D, a.T) ||
+        !make_store_map(&tm_g, a.G, a.V, a.D))
+        return cudaErrorInvalidValue;
     // per device and cheap: set on every call
-    cudaError_t e = cudaFuncSetAttribute(k_lmhead_grad<CL>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    cudaError_t e = cudaFuncSetAttribute(k_lmhead_grad, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kLmSmemBytes);
     if (e != cudaSuccess)
         return e;
@@ -696,38 +679,25 @@ cudaError_t launch_cl(const CUtensorMap &tm_dl, const CUtensorMap &tm_h, const C
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = CL;
+    attr[0].val.clusterDim.x = 2;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    // persistent: as many clusters as fit on the GPU at once (clusters are
-    // placed within one GPC, so this can be below kSms / CL)
+    // persistent: as many pairs as fit on the GPU at once
     cfg.gridDim = dim3(kSms);
     int fit = 0;
-    e = cudaOccupancyMaxActiveClusters(&fit, k_lmhead_grad<CL>, &cfg);
+    e = cudaOccupancyMaxActiveClusters(&fit, k_lmhead_grad, &cfg);
     if (e != cudaSuccess)
         return e;
     if (fit < 1)
         return cudaErrorInvalidConfiguration;
-    const int groups = (lmhead_row_blocks(a.V) + CL - 1) / CL * lmhead_col_blocks(a.D);
-    const int nclusters = groups < fit ? groups : fit;
-    cfg.gridDim = dim3(nclusters * CL);
+    const int pairs = (lmhead_row_blocks(a.V) + 1) / 2 * lmhead_col_blocks(a.D);
+    const int nclusters = pairs < fit ? pairs : fit;
+    cfg.gridDim = dim3(nclusters * 2);
     const int band = kLmBand < lmhead_col_blocks(a.D) ? kLmBand : lmhead_col_blocks(a.D);
-    return cudaLaunchKernelEx(&cfg, k_lmhead_grad<CL>, tm_dl, tm_h, tm_g, colpart, rowpart, flags, (int)a.V,
+    return cudaLaunchKernelEx(&cfg, k_lmhead_grad, tm_dl, tm_h, tm_g, colpart, rowpart, flags, (int)a.V,
                               (int)a.D, (int)a.T, band);
-}
-
-}  // namespace
-
-cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
-                               cudaStream_t stream)
-{
-    CUtensorMap tm_dl, tm_h, tm_g;
-    if (!make_map(&tm_dl, a.dlogits, a.V, a.T) || !make_map(&tm_h, a.hidden, a.D, a.T) ||
-        !make_store_map(&tm_g, a.G, a.V, a.D))
-        return cudaErrorInvalidValue;
-    return launch_cl<kLmCluster>(tm_dl, tm_h, tm_g, a, colpart, rowpart, flags, stream);
 }
 
 }  // namespace ember

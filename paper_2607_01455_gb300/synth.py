@@ -69,6 +69,8 @@ WORKLOADS = {
         Workload("dense_lmhead_v128256_d8192_bf16", 128256, 8192, "bf16", 50, heavy_frac=0.01),
         Workload("lmhead_grad_v128256_d8192_t4096_bf16", 128256, 8192, "bf16", 20, kind="lmhead",
                  T=4096),
+        # a quarter of the head's rows: the size the detailed profiles use
+        Workload("lmhead_grad_v32768_d8192_t4096_bf16", 32768, 8192, "bf16", 20, kind="lmhead", T=4096),
     ]
 }
 # The five workloads of the optimizer step in the order they are listed for
