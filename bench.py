@@ -36,6 +36,10 @@ L2_FLUSH_BYTES = 512 << 20
 # capture summarised in profiles/dense_lmhead_v128256_d8192_bf16_launches.md.
 # Set to None whenever k_apply_dense changes until it is captured again.
 APPLY_TRAFFIC_BYTES = 8374871296
+# The same for k_lmhead_grad on the LM-head gradient workload (V=128256,
+# D=8192, T=4096), from profiles/lmhead_grad_v128256_d8192_t4096_bf16_launches.md.
+# Set to None whenever k_lmhead_grad changes until it is captured again.
+LMHEAD_TRAFFIC_BYTES = {"lmhead_grad_v128256_d8192_t4096_bf16": 11450829184}
 
 
 def wbytes(wl):
@@ -257,7 +261,8 @@ def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
             "roofline": {"bound": "tensor", "kernel": "k_lmhead_grad", "achieved": tf, "peak": peaks["burst"],
                          "unit": "TFLOP/s", "frac": tf / peaks["burst"],
                          "frac_of_sustained": tf / peaks["sustained"], "peak_kind": peak_kind,
-                         "flops_per_launch": flops, "traffic": None},
+                         "flops_per_launch": flops, "traffic": LMHEAD_TRAFFIC_BYTES.get(wl.name),
+                         "algorithmic_dram_bytes_per_launch": 2 * T * (V + D) + 4 * V * D},
             "unfused": {"ms_per_step": ms_unfused, "cublas_gemm_ms": ms_cublas, "cublas_tflops": tf_cublas,
                         "cublas_output": cublas_out,
                         "what": "torch.mm(dlogits^T, H) then ember_step_dense (reduce, state, apply)"},
