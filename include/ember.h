@@ -197,6 +197,48 @@ ember_status ember_lmhead_grad(ember_handle *h, const void *dlogits, const void 
 ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, const void *hidden,
                                int64_t T, float *G, float *state, float lr, int64_t t, void *stream);
 
+/* Row-sharded dense step (Section 2.3: the statistics are sums of g^2, so
+ * a table whose rows are spread over ranks needs only the per-rank partial
+ * sums exchanged before the update).  A step is two calls per shard with
+ * one exchange between them:
+ *
+ *   ember_shard_reduce  (every shard)  the reduction pass over the shard's
+ *       rows: updates r for those rows and writes the shard's exchange block
+ *       (its per-CTA column sums of g^2 and sums of new r);
+ *   the caller all-gathers the blocks in shard order (NCCL all_gather of
+ *       ember_shard_exchange_bytes per shard, or any copy);
+ *   ember_shard_update  (every shard)  the column EMA and normaliser from all
+ *       blocks (every shard forms the same c and s), then the update of the
+ *       shard's rows of W.
+ *
+ * Shards are cut at the boundaries of the whole-table step's fixed CTA row
+ * ranges, and every per-CTA partial is formed by the same kernel over the
+ * same rows, so W, r and c come out bit-identical to ember_step_dense for
+ * any number of shards (the paper's "bitwise identical" requirement of
+ * Section 2.3).  The exchange holds one partial row per CTA (at most 304 x
+ * D floats in all) rather than one reduced row, which is what keeps the
+ * sum order independent of the shard count.
+ *
+ *   shard, nshards: 0 <= shard < nshards <= 4096.  Shards past the table's
+ *       last CTA hold no rows (their calls still take part: the update
+ *       maintains c).
+ *   G_shard, W_shard: the shard's rows (ember_shard_rows), row-major,
+ *       device memory; with D % 4 == 0 they must be 16-byte aligned (8-byte
+ *       for bf16 W) so that every shard takes the whole-table step's
+ *       vector path (EMBER_ERR_ALIGNMENT otherwise).
+ *   state: a full V + D buffer per shard; only the shard's rows of r and all
+ *       of c are read and written.
+ *   block: ember_shard_exchange_bytes(h, nshards) bytes, device, 256-byte
+ *       aligned; blocks: nshards of them back to back, in shard order.
+ * Variant ROW is not offered (EMBER_ERR_UNSUPPORTED): its one-pass kernel
+ * needs no exchange for W and is run per shard with ember_step_dense. */
+int64_t ember_shard_rows(const ember_handle *h, int shard, int nshards, int64_t *row0);
+size_t ember_shard_exchange_bytes(const ember_handle *h, int nshards);
+ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const float *G_shard, float *state,
+                                void *block, void *stream);
+ember_status ember_shard_update(ember_handle *h, int shard, int nshards, void *W_shard, const float *G_shard,
+                                float *state, const void *blocks, float lr, int64_t t, void *stream);
+
 /* One sparse Ember step (Section 2.2) at step number t >= 1.
  *   ids:   N token ids of type idtype (duplicates allowed, any order).
  *   rows:  N x D fp32, row k is the gradient contribution of occurrence k

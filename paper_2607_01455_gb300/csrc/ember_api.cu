@@ -24,7 +24,7 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
     };
     const size_t nstate = (size_t)((D + kStateCols - 1) / kStateCols);
     L.scalars = take(sizeof(DevScalars));
-    L.rsum_part = take(sizeof(double) * kGridCtas);
+    L.rsum_part = take(sizeof(double) * kRsumParts);
     L.csum_part = take(sizeof(double) * nstate);
     L.colpart = take(sizeof(float) * (size_t)kPartRows * (size_t)D);
     if (max_sparse_N > 0) {
@@ -311,6 +311,127 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
     const bool vec4 = is_aligned(W, 4 * wsz);  // D % 8 == 0 and G 16-byte aligned already
     if (!choose_colmap(h->D, vec4, &a.map))
         return EMBER_ERR_UNSUPPORTED;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+// ---- row-sharded dense step ----
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+static bool shard_plan(const ember_handle *h, int shard, int nshards, ShardArgs *p)
+{
+    if (!h || nshards < 1 || nshards > kMaxShards || shard < 0 || shard >= nshards)
+        return false;
+    const int nparts = dense_parts(h->V);
+    const int cap = (nparts + nshards - 1) / nshards;
+    int b0 = shard * cap, b1 = (shard + 1) * cap;
+    if (b0 > nparts)
+        b0 = nparts;
+    if (b1 > nparts)
+        b1 = nparts;
+    p->cta_begin = b0;
+    p->cta_end = b1;
+    p->cap = cap;
+    p->nshards = nshards;
+    p->row_base = (int64_t)b0 * h->V / nparts;
+    p->block_rsum = align256(sizeof(float) * (size_t)cap * (size_t)h->D);
+    p->block_bytes = p->block_rsum + align256(sizeof(double) * (size_t)cap);
+    return true;
+}
+
+int64_t ember_shard_rows(const ember_handle *h, int shard, int nshards, int64_t *row0)
+{
+    ShardArgs p{};
+    if (!shard_plan(h, shard, nshards, &p))
+        return -1;
+    const int nparts = dense_parts(h->V);
+    const int64_t r1 = (int64_t)p.cta_end * h->V / nparts;
+    if (row0)
+        *row0 = p.row_base;
+    return r1 - p.row_base;
+}
+
+size_t ember_shard_exchange_bytes(const ember_handle *h, int nshards)
+{
+    ShardArgs p{};
+    if (!shard_plan(h, 0, nshards, &p))
+        return 0;
+    return p.block_bytes;
+}
+
+static ember_status shard_common(ember_handle *h, int shard, int nshards, const void *W_shard, const float *G_shard,
+                                 const float *state, const void *block, ShardArgs *p, DenseArgs *a)
+{
+    if (!h || !state || !block)
+        return EMBER_ERR_INVALID_ARG;
+    if (!shard_plan(h, shard, nshards, p))
+        return EMBER_ERR_INVALID_ARG;
+    const bool has_rows = p->cta_end > p->cta_begin;
+    if (has_rows && !G_shard)
+        return EMBER_ERR_INVALID_ARG;
+    if (h->hp.variant == EMBER_VARIANT_ROW)
+        return EMBER_ERR_UNSUPPORTED;  // the row-only step has its own one-pass kernel
+    // every shard must take the same vector path as the whole-table step
+    const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
+    const bool vec4 = h->D % 4 == 0;
+    if (!is_aligned(state, 4) || !is_aligned(block, 256) ||
+        (has_rows && (!is_aligned(G_shard, vec4 ? 16 : 4) || (W_shard && !is_aligned(W_shard, vec4 ? 4 * wsz : wsz)))))
+        return EMBER_ERR_ALIGNMENT;
+    if (!h->ws)
+        return EMBER_ERR_WORKSPACE;
+    a->V = h->V;
+    a->D = h->D;
+    a->wbf16 = h->wdtype == EMBER_BF16;
+    a->G = G_shard;
+    a->r = const_cast<float *>(state);
+    a->c = const_cast<float *>(state) + h->V;
+    a->beta2 = h->hp.beta2;
+    a->one_minus_beta2 = 1.0 - h->hp.beta2;
+    a->eps = (float)h->hp.eps;
+    a->variant = h->hp.variant;
+    a->ws = h->ws;
+    a->lay = make_layout(h->V, h->D, h->ws_max_N);
+    a->trace = nullptr;
+    if (!choose_colmap(h->D, vec4, &a->map))
+        return EMBER_ERR_UNSUPPORTED;
+    return EMBER_OK;
+}
+
+ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const float *G_shard, float *state,
+                                void *block, void *stream)
+{
+    ShardArgs p{};
+    DenseArgs a{};
+    const ember_status st = shard_common(h, shard, nshards, nullptr, G_shard, state, block, &p, &a);
+    if (st != EMBER_OK)
+        return st;
+    p.phase = 1;
+    p.block = block;
+    a.shard = &p;
+    a.inv_bc = 1.0;
+    a.stream = (cudaStream_t)stream;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+ember_status ember_shard_update(ember_handle *h, int shard, int nshards, void *W_shard, const float *G_shard,
+                                float *state, const void *blocks, float lr, int64_t t, void *stream)
+{
+    if (t < 1 || !isfinite(lr))
+        return EMBER_ERR_INVALID_ARG;
+    ShardArgs p{};
+    DenseArgs a{};
+    a.W = W_shard;
+    const ember_status st = shard_common(h, shard, nshards, W_shard, G_shard, state, blocks, &p, &a);
+    if (st != EMBER_OK)
+        return st;
+    if (p.cta_end > p.cta_begin && !W_shard)
+        return EMBER_ERR_INVALID_ARG;
+    p.phase = 2;
+    p.blocks = blocks;
+    a.shard = &p;
+    a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
+    a.lr_signed = h->hp.maximize ? lr : -lr;
+    a.stream = (cudaStream_t)stream;
     return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
 }
 

@@ -49,7 +49,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                float *__restrict__ colpart, double *__restrict__ rsum_part,
                int64_t V, int D, int tpr, double beta2, double one_minus_beta2,
-               float *__restrict__ G_stage)
+               float *__restrict__ G_stage, RowSpan span)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
@@ -61,8 +61,8 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     const int g = tid / tpr;                 // this thread's row group
     const int l = tid - g * tpr;             // position within the row
     const int wpg = tpr >> 5;                // warps per row group
-    const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
-    const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+    const int64_t row0 = (int64_t)(span.cta_base + blockIdx.x) * V / span.nparts;
+    const int64_t row1 = (int64_t)(span.cta_base + blockIdx.x + 1) * V / span.nparts;
 
     grid_dep_wait();    // the first kernel of a step: returns at once
     grid_dep_launch();  // the state pass may start launching now; it waits for this grid
@@ -94,12 +94,13 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                 const int col = l + c * tpr;
                 const bool in = i < row1 && col < DV;
                 if constexpr (STAGE) {
-                    const int64_t idx = i * D + (int64_t)col * VEC;
+                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
                     v[k][c] = in ? *reinterpret_cast<const F *>(G + idx) : zero_vec<VEC>();
                     if (in)
                         *reinterpret_cast<F *>(G_stage + idx) = v[k][c];
                 } else {
-                    v[k][c] = in ? load_g<VEC>(G + i * D + (int64_t)col * VEC) : zero_vec<VEC>();
+                    v[k][c] = in ? load_g<VEC>(G + (i - span.row_base) * D + (int64_t)col * VEC)
+                                 : zero_vec<VEC>();
                 }
             }
         }
@@ -354,7 +355,8 @@ template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__restrict__ r,
               const float *__restrict__ c, const DevScalars *__restrict__ sc,
-              int64_t V, int D, int tpr, float inv_bc, float eps, float lr_signed, int variant)
+              int64_t V, int D, int tpr, float inv_bc, float eps, float lr_signed, int variant,
+              RowSpan span)
 {
     using F = typename Vec<VEC>::F;
     using WT = typename WRaw<BF16, VEC>::T;
@@ -364,8 +366,8 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
     const int rg = kThreads / tpr;
     const int g = tid / tpr;
     const int l = tid - g * tpr;
-    const int64_t row0 = (int64_t)blockIdx.x * V / gridDim.x;
-    const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+    const int64_t row0 = (int64_t)(span.cta_base + blockIdx.x) * V / span.nparts;
+    const int64_t row1 = (int64_t)(span.cta_base + blockIdx.x + 1) * V / span.nparts;
     const int64_t step = (int64_t)rg * R;
     const int64_t nblocks = (row1 - row0 + step - 1) / step;
 
@@ -378,7 +380,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (i < row1 && col < DV) {
-                    const int64_t idx = i * D + (int64_t)col * VEC;
+                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
                     asm volatile("prefetch.global.L2 [%0];" ::"l"(G + idx));
                     asm volatile("prefetch.global.L2 [%0];" ::"l"(static_cast<const char *>(W) +
                                                                    idx * (BF16 ? 2 : 4)));
@@ -406,8 +408,9 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (i < row1 && col < DV) {
-                    gv[k][cc] = load_g<VEC>(G + i * D + (int64_t)col * VEC);
-                    wr[k][cc] = load_w<BF16, VEC>(W, i * D + (int64_t)col * VEC);
+                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
+                    gv[k][cc] = load_g<VEC>(G + idx);
+                    wr[k][cc] = load_w<BF16, VEC>(W, idx);
                 }
             }
         }
@@ -430,7 +433,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
                     const float u = comp(gv[k][cc], e) / den;
                     w[e] = fmaf(lr_signed, u, w[e]);
                 }
-                store_w<BF16, VEC>(W, i * D + (int64_t)col * VEC, w);
+                store_w<BF16, VEC>(W, (i - span.row_base) * D + (int64_t)col * VEC, w);
             }
         }
     }
@@ -590,12 +593,33 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
     }
 }
 
+// Row-sharded step: copy the per-CTA partials of every shard's exchange
+// block (CTA b is entry b % cap of shard b / cap) into the workspace layout
+// of the whole-table step, in CTA order.
+__global__ void k_shard_unpack(const unsigned char *__restrict__ blocks, size_t block_bytes, size_t block_rsum,
+                               int cap, int nparts, int D, float *__restrict__ colpart,
+                               double *__restrict__ rsum_part)
+{
+    grid_dep_wait();
+    grid_dep_launch();
+    const int64_t total = (int64_t)nparts * D;
+    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total;
+         q += (int64_t)gridDim.x * blockDim.x) {
+        const int b = (int)(q / D);
+        const int j = (int)(q - (int64_t)b * D);
+        const float *src = reinterpret_cast<const float *>(blocks + (size_t)(b / cap) * block_bytes);
+        colpart[q] = src[(int64_t)(b % cap) * D + j];
+    }
+    for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < nparts; b += gridDim.x * blockDim.x)
+        rsum_part[b] = reinterpret_cast<const double *>(blocks + (size_t)(b / cap) * block_bytes + block_rsum)[b % cap];
+}
+
 template <int VEC, int CPT>
 cudaError_t launch_dense_t(const DenseArgs &a)
 {
     constexpr int R1 = (16 / CPT) < 1 ? 1 : (16 / CPT);
     constexpr int R3 = (8 / CPT) < 1 ? 1 : (8 / CPT);
-    const int nparts = (int)(a.V < kGridCtas ? a.V : kGridCtas);
+    const int nparts = dense_parts(a.V);
     const int D = (int)a.D;
     DevScalars *sc = reinterpret_cast<DevScalars *>(a.ws + a.lay.scalars);
     double *rsum_part = reinterpret_cast<double *>(a.ws + a.lay.rsum_part);
@@ -609,6 +633,42 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     // dependent launch.
     const bool pdl = (a.trace == nullptr);
     cudaError_t e;
+    RowSpan span{0, nparts, 0};
+    if (a.shard) {
+        // one phase of a row-sharded step: the shard's own CTAs of the
+        // whole-table grid, so each per-CTA partial equals the unsharded one
+        const ShardArgs &sh = *a.shard;
+        const int ncta = sh.cta_end - sh.cta_begin;
+        span = RowSpan{sh.cta_begin, nparts, sh.row_base};
+        if (sh.phase == 1) {
+            if (ncta == 0)
+                return cudaSuccess;
+            float *bcol = static_cast<float *>(sh.block);
+            double *brsum = reinterpret_cast<double *>(static_cast<unsigned char *>(sh.block) + sh.block_rsum);
+            e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(ncta), dim3(kThreads), shmem, a.stream, false,
+                         a.G, a.r, bcol, brsum, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr, span);
+            return e != cudaSuccess ? e : cudaGetLastError();
+        }
+        e = launch_k(k_shard_unpack, dim3(kGridCtas), dim3(kThreads), 0, a.stream, false,
+                     static_cast<const unsigned char *>(sh.blocks), sh.block_bytes, sh.block_rsum, sh.cap, nparts, D,
+                     colpart, rsum_part);
+        if (e != cudaSuccess)
+            return e;
+        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        if (e != cudaSuccess || ncta == 0)
+            return e != cudaSuccess ? e : cudaGetLastError();
+        const size_t cs_bytes = (size_t)D * sizeof(float);
+        if (a.wbf16)
+            e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.variant, span);
+        else
+            e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.variant, span);
+        return e != cudaSuccess ? e : cudaGetLastError();
+    }
     if (a.variant == EMBER_VARIANT_ROW && !a.lm) {
         // one pass over G and W, then the column state; no apply pass
         constexpr int RR = (4 / CPT) < 1 ? 1 : (4 / CPT);
@@ -651,7 +711,8 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             cudaEventRecord(a.trace[1], a.stream);
         // plain stream order after the tensor-core kernel: launched early,
         // the state grid made the step slower (measured 0.1-0.3 ms)
-        const int nrow_ctas = kSms;
+        const int64_t vb = (a.V + kStateThreads - 1) / kStateThreads;
+        const int nrow_ctas = (int)(vb < kMaxRowCtas ? vb : kMaxRowCtas);
         e = launch_state(lm_col, lmhead_row_blocks(a.V), rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D,
                          a.beta2, a.one_minus_beta2, a.inv_bc, a.stream, false, a.r, nullptr, lm_row,
                          lmhead_col_blocks(a.D), nrow_ctas);
@@ -662,10 +723,10 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             cudaEventRecord(a.trace[0], a.stream);
         if (a.G_stage)
             e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage);
+                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage, span);
         else
             e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr);
+                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr, span);
         if (e != cudaSuccess)
             return e;
         if (a.trace)
@@ -683,11 +744,11 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     if (a.wbf16)
         e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
                      a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
-                     a.eps, a.lr_signed, a.variant);
+                     a.eps, a.lr_signed, a.variant, span);
     else
         e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
                      a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
-                     a.eps, a.lr_signed, a.variant);
+                     a.eps, a.lr_signed, a.variant, span);
     if (e != cudaSuccess)
         return e;
     if (a.trace)

@@ -24,9 +24,12 @@ constexpr int kSparseCtasPerSm = 3;
 constexpr int kSparseCtas = kSms * kSparseCtasPerSm;
 constexpr int kPartRows = kSparseCtas > kGridCtas ? kSparseCtas : kGridCtas;
 
-// The state pass reduces 32 columns per CTA.
+// The state pass reduces 32 columns per CTA; its row pass (sparse and LM-head
+// steps) runs up to kMaxRowCtas CTAs, so that a thread has about one row.
 constexpr int kStateCols = 32;
 constexpr int kStateThreads = 256;
+constexpr int kMaxRowCtas = 1024;
+constexpr int kRsumParts = kMaxRowCtas > kGridCtas ? kMaxRowCtas : kGridCtas;
 
 // Bits of the sticky device flag.
 constexpr unsigned kFlagIdRange = 1u << 0;
@@ -53,7 +56,7 @@ constexpr int kSortThreads = 256;
 // Workspace layout (byte offsets, each 256-byte aligned).
 struct Layout {
     size_t scalars;     // DevScalars
-    size_t rsum_part;   // double[kGridCtas]            sum of new r per CTA
+    size_t rsum_part;   // double[kRsumParts]           sum of new r per CTA
     size_t csum_part;   // double[ceil(D/32)]           sum of new c per state CTA
     size_t colpart;     // float[kPartRows * D]     column sums of g^2 per CTA
     // sparse step (present when max_sparse_N > 0); N = max_sparse_N,
@@ -105,6 +108,32 @@ int lmhead_col_blocks(int64_t D);
 cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, unsigned *flags,
                                cudaStream_t stream);
 
+// Rows a launch of the reduce or apply kernel covers: its CTA b is CTA
+// cta_base + b of a grid of nparts over the whole table (row range
+// [(cta_base+b) V / nparts, (cta_base+b+1) V / nparts)), and the G and W
+// pointers hold rows from row_base on.  The whole-table step uses
+// {0, nparts, 0}; a row shard uses its own CTAs of the same grid, so every
+// per-CTA partial is the one the whole-table step would form.
+struct RowSpan {
+    int cta_base;
+    int nparts;
+    int64_t row_base;
+};
+
+// Row-sharded dense step (see ember_shard_reduce / ember_shard_update).
+constexpr int kMaxShards = 4096;
+struct ShardArgs {
+    int phase;            // 1: reduce and write this shard's exchange block; 2: state and apply
+    int cta_begin, cta_end;
+    int cap;              // CTAs per shard block (the last shard may use fewer)
+    int nshards;
+    int64_t row_base;     // first row this shard holds
+    void *block;          // phase 1: this shard's exchange block
+    const void *blocks;   // phase 2: every shard's block, in shard order
+    size_t block_bytes;
+    size_t block_rsum;    // offset of the fp64 row sums inside a block
+};
+
 struct DenseArgs {
     int64_t V, D;
     int wbf16;
@@ -123,7 +152,11 @@ struct DenseArgs {
     const cudaEvent_t *trace;  // nullptr, or events[0..3] to record at kernel boundaries
     float *G_stage;            // nullptr, or the HBM copy the reduce pass writes of a host-resident G
     const LmArgs *lm;          // nullptr, or: G is formed by the LM-head kernel instead of read
+    const ShardArgs *shard;    // nullptr, or: one phase of a row-sharded step
 };
+
+// CTAs of the dense step's reduce and apply grids for a V-row table.
+inline int dense_parts(int64_t V) { return (int)(V < kGridCtas ? V : kGridCtas); }
 
 cudaError_t launch_dense_step(const DenseArgs &a);
 

@@ -39,6 +39,7 @@ EXPORTS = (
     "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
     "ember_step_dense_noalloc", "ember_step_dense_from_host",
     "ember_lmhead_grad", "ember_step_lmhead",
+    "ember_shard_rows", "ember_shard_exchange_bytes", "ember_shard_reduce", "ember_shard_update",
 )
 
 
@@ -87,6 +88,10 @@ def lib():
             "ember_step_dense_from_host": (st, [vp, vp, vp, vp, vp, flt, i64, vp]),
             "ember_lmhead_grad": (st, [vp, vp, vp, i64, vp, vp]),
             "ember_step_lmhead": (st, [vp, vp, vp, vp, i64, vp, vp, flt, i64, vp]),
+            "ember_shard_rows": (i64, [vp, ip, ip, ctypes.POINTER(i64)]),
+            "ember_shard_exchange_bytes": (sz, [vp, ip]),
+            "ember_shard_reduce": (st, [vp, ip, ip, vp, vp, vp, vp]),
+            "ember_shard_update": (st, [vp, ip, ip, vp, vp, vp, vp, flt, i64, vp]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -186,6 +191,29 @@ def ember_step_lmhead(h, W, dlogits, hidden, T, G, state, lr, t, stream=None):
                                    lr, t, _stream(stream)), "ember_step_lmhead")
 
 
+def ember_shard_rows(h, shard, nshards):
+    """(row0, rows) that shard `shard` of `nshards` holds."""
+    row0 = ctypes.c_int64(0)
+    n = lib().ember_shard_rows(h, shard, nshards, ctypes.byref(row0))
+    if n < 0:
+        raise EmberError(EMBER_ERR_INVALID_ARG, "ember_shard_rows")
+    return row0.value, n
+
+
+def ember_shard_exchange_bytes(h, nshards):
+    return lib().ember_shard_exchange_bytes(h, nshards)
+
+
+def ember_shard_reduce(h, shard, nshards, G_shard, state, block, stream=None):
+    _check(lib().ember_shard_reduce(h, shard, nshards, _addr(G_shard), _addr(state), _addr(block),
+                                    _stream(stream)), "ember_shard_reduce")
+
+
+def ember_shard_update(h, shard, nshards, W_shard, G_shard, state, blocks, lr, t, stream=None):
+    _check(lib().ember_shard_update(h, shard, nshards, _addr(W_shard), _addr(G_shard), _addr(state),
+                                    _addr(blocks), lr, t, _stream(stream)), "ember_shard_update")
+
+
 def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
     _check(lib().ember_step_sparse(h, _addr(W), _addr(ids), idtype, N, _addr(rows), _addr(state),
                                    lr, t, _stream(stream)), "ember_step_sparse")
@@ -257,6 +285,20 @@ class Ember:
     def step_lmhead(self, W, dlogits, hidden, G, lr, t, stream=None):
         """One step of an LM head whose gradient dlogits^T hidden is formed into G."""
         ember_step_lmhead(self.handle, W, dlogits, hidden, dlogits.shape[0], G, self.state, lr, t, stream)
+
+    # row-sharded dense step: this object is one shard's rank (its own
+    # state and workspace); see include/ember.h for the protocol
+    def shard_rows(self, shard, nshards):
+        return ember_shard_rows(self.handle, shard, nshards)
+
+    def shard_exchange_bytes(self, nshards):
+        return ember_shard_exchange_bytes(self.handle, nshards)
+
+    def shard_reduce(self, shard, nshards, G_shard, block, stream=None):
+        ember_shard_reduce(self.handle, shard, nshards, G_shard, self.state, block, stream)
+
+    def shard_update(self, shard, nshards, W_shard, G_shard, blocks, lr, t, stream=None):
+        ember_shard_update(self.handle, shard, nshards, W_shard, G_shard, self.state, blocks, lr, t, stream)
 
     def step_sparse(self, W, ids, rows, lr, t, stream=None):
         import torch
