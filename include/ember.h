@@ -108,10 +108,13 @@ size_t ember_state_numel(const ember_handle *h);
 /* Bytes of device workspace the steps of this handle need when sparse steps
  * carry at most max_sparse_N ids (0 if only dense steps are used).  Returns
  * 0 for a NULL handle or a negative max_sparse_N.  The workspace holds
- * per-block partial sums, the sort buffers of the sparse step, the summed
- * gradient rows of the sparse step (up to max_sparse_N x D fp32) and a few
- * scalars; it is not optimizer state and need not persist between steps,
- * but the caller must not touch it while a step is in flight. */
+ * per-block partial sums (among them the LM-head step's per-tile sums of
+ * g^2, V*D*4*(1/128 + 1/256) bytes, always reserved), the sort buffers of
+ * the sparse step, the summed gradient rows of the sparse step (up to
+ * max_sparse_N x D fp32), a V-entry map of touched rows and a few scalars.
+ * It is not optimizer state, but the steps leave the touched-row map zeroed
+ * for the next one: the caller must not write to the workspace after binding
+ * it, nor touch it while a step is in flight. */
 size_t ember_workspace_bytes(const ember_handle *h, int64_t max_sparse_N);
 
 /* Give the handle its device workspace (256-byte aligned, at least
