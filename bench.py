@@ -92,7 +92,8 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
     ids, rows = synth.sparse_batch(wl, seed, 1, dev)
     U = int(torch.unique(ids).numel())
     emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, max_sparse_N=wl.N, device=dev)
-    nk = len(SPARSE_KERNELS)
+    names = SPARSE_KERNELS
+    nk = len(names)
     t = 0
     warm = [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)]
     for i in range(warmup):
@@ -120,7 +121,7 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
         raise SystemExit("device status after the sparse steps")
     plain = [k for k in range(steps) if k not in kern_ev]
     per = {name: sum(kern_ev[k][i].elapsed_time(kern_ev[k][i + 1]) for k in traced) / len(traced)
-           for i, name in enumerate(SPARSE_KERNELS)}
+           for i, name in enumerate(names)}
     ms = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain)
     ms_traced = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in traced) / len(traced)
     # the same step replayed from a CUDA graph (how a training loop would run it)

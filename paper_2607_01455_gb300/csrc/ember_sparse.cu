@@ -453,8 +453,15 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
         const bool last_cut = p1 < n_valid && segidx[p1] == u_last;
         int cur = u_first;
         int len = 0;  // occurrences of `cur` seen in this range
+        // Per-id sums in occurrence order, compensated (Kahan): `acc` is the
+        // running sum, `cmp` the part of it that rounding added, so the sum
+        // stays within about an ulp even over thousands of duplicates.
         F acc = zero_vec<VEC>();
+        F cmp = zero_vec<VEC>();
         auto flush = [&](int u) {
+#pragma unroll
+            for (int e = 0; e < VEC; ++e)
+                set_comp(acc, e, comp(acc, e) - comp(cmp, e));
             const bool before = first_cut && u == u_first;
             const bool after = last_cut && u == u_last;
             if (!before && !after) {
@@ -516,13 +523,18 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                     if (uu[k] != cur) {
                         flush(cur);
                         acc = zero_vec<VEC>();
+                        cmp = zero_vec<VEC>();
                         cur = uu[k];
                         len = 0;
                     }
                     ++len;
 #pragma unroll
-                    for (int e = 0; e < VEC; ++e)
-                        set_comp(acc, e, comp(acc, e) + comp(v[k], e));
+                    for (int e = 0; e < VEC; ++e) {
+                        const float y = comp(v[k], e) - comp(cmp, e);
+                        const float t = comp(acc, e) + y;
+                        set_comp(cmp, e, (t - comp(acc, e)) - y);
+                        set_comp(acc, e, t);
+                    }
                 }
             }
         }
@@ -586,6 +598,7 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
         if (active) {
             const int64_t off = (int64_t)col * VEC;
             F acc = load_g<VEC>(carry + ((int64_t)2 * w0 + 1) * D + off);
+            F cmp = zero_vec<VEC>();  // compensated (Kahan) sum, as in k_sp_segsum
             constexpr int kB = 8;
             for (int qb = w0 + 1; qb <= w1; qb += kB) {
                 F v[kB];
@@ -598,9 +611,16 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
 #pragma unroll
                 for (int k = 0; k < kB; ++k)
 #pragma unroll
-                    for (int e = 0; e < VEC; ++e)
-                        set_comp(acc, e, comp(acc, e) + comp(v[k], e));
+                    for (int e = 0; e < VEC; ++e) {
+                        const float y = comp(v[k], e) - comp(cmp, e);
+                        const float t = comp(acc, e) + y;
+                        set_comp(cmp, e, (t - comp(acc, e)) - y);
+                        set_comp(acc, e, t);
+                    }
             }
+#pragma unroll
+            for (int e = 0; e < VEC; ++e)
+                set_comp(acc, e, comp(acc, e) - comp(cmp, e));
             *reinterpret_cast<F *>(S + (int64_t)u * D + off) = acc;
 #pragma unroll
             for (int e = 0; e < VEC; ++e) {

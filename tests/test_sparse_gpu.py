@@ -67,9 +67,12 @@ def check_dedup(emb, ids):
     np.testing.assert_array_equal(counts.cpu().numpy(), want_c)
 
 
+# 1024-key sort tiles: 4096, 4097, 32768 and 32769 sit on tile edges; the
+# largest batches span 64 tiles.
 @pytest.mark.parametrize("V,D,N", [
     (50, 8, 1), (50, 8, 37), (1000, 64, 4096), (1000, 64, 4097), (5000, 200, 9000),
     (3000, 203, 5000), (262144, 128, 12288), (100, 2048, 3000), (20000, 8192, 700),
+    (262144, 8, 32768), (7, 8, 32768), (70000, 8, 32769), (5000, 8, 65536), (300000, 16, 50000),
 ])
 @pytest.mark.parametrize("idtype", [torch.int64, torch.int32])
 def test_dedup_bit_exact(cuda_device, V, D, N, idtype):
@@ -171,6 +174,27 @@ def test_sparse_edge_cases(cuda_device):
     with pytest.raises(EmberError) as ex:
         emb.step_sparse(W, big, torch.zeros(20001, D, device=cuda_device), 1e-3, t + 1)
     assert ex.value.status == EMBER_ERR_WORKSPACE
+
+
+def test_skipped_ids_leave_the_step_bit_identical(cuda_device):
+    """The same batch, and the batch followed by 10000 skipped ids (id -1,
+    whose rows are never read), give bit-identical W and state: skipped ids
+    sort after every valid one, so the segment sums see the same order."""
+    V, D, N, Npad = 20000, 256, 30000, 40000
+    ids, rows = batch(V, D, N, 1, cuda_device, seed=11)
+    ids_pad = torch.cat([ids, torch.full((Npad - N,), -1, dtype=ids.dtype, device=cuda_device)])
+    rows_pad = torch.cat([rows, torch.full((Npad - N, D), float("nan"), device=cuda_device)])
+    outs = []
+    for i, r in ((ids, rows), (ids_pad, rows_pad)):
+        emb = make(V, D, "bf16", Npad)
+        W = (torch.randn(V, D, device=cuda_device, generator=torch.Generator(device=cuda_device)
+                         .manual_seed(3)) * 0.02).to(torch.bfloat16)
+        for t in (1, 2):
+            emb.step_sparse(W, i, r, 1e-3, t)
+        outs.append((W, emb.state.clone(), emb.device_status()))
+    assert outs[0][2] == 0 and outs[1][2] == EMBER_ERR_ID_OUT_OF_RANGE
+    assert torch.equal(outs[0][0].view(torch.int16), outs[1][0].view(torch.int16))
+    assert torch.equal(outs[0][1].view(torch.int32), outs[1][1].view(torch.int32))
 
 
 def test_sparse_v1_and_tiny(cuda_device):
