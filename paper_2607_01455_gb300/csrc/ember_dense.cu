@@ -234,6 +234,9 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
     const int nstate = (int)gridDim.x - rowp.nrow_ctas;
     __shared__ double part[kW][32];
     __shared__ bool am_last;
+    // means as products: fp64 division is a long instruction sequence, and
+    // the row pass of a sparse step runs it for every row of the table
+    const double inv_D = 1.0 / (double)D, inv_V = 1.0 / (double)V;
     grid_dep_wait();  // column partials and row sums of the earlier passes
     grid_dep_launch();
 
@@ -267,7 +270,7 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
                 tot += part[q][lane];
             double cn = 0.0;
             if (j < D) {
-                const double mean_col = tot / (double)V;
+                const double mean_col = tot * inv_V;
                 const float cnew = (float)(beta2 * (double)c[j] + one_minus_beta2 * mean_col);
                 c[j] = cnew;
                 cn = (double)cnew;
@@ -280,28 +283,52 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
         }
     } else {
         const int rb = (int)blockIdx.x - nstate;
+        const int64_t stride = (int64_t)rowp.nrow_ctas * kStateThreads;
         double rsum = 0.0;
-        for (int64_t i = (int64_t)rb * kStateThreads + threadIdx.x; i < V;
-             i += (int64_t)rowp.nrow_ctas * kStateThreads) {
-            double mean_row = 0.0;
-            if (rowp.slot == nullptr) {
-                // every row: per-column-block sums, slice-major, in block order
+        if (rowp.slot == nullptr) {
+            // every row: per-column-block sums, slice-major, in block order
+            for (int64_t i = (int64_t)rb * kStateThreads + threadIdx.x; i < V; i += stride) {
                 float tot = 0.f;
 #pragma unroll 8
                 for (int k = 0; k < rowp.nslices; ++k)
                     tot += __ldcg(rowp.rowpart + (int64_t)k * V + i);
-                mean_row = (double)tot / (double)D;
-            } else if (const int sl = rowp.slot[i]) {
-                const int64_t u = sl - 1;
-                float tot = 0.f;
-                for (int k = 0; k < rowp.nslices; ++k)
-                    tot += rowp.rowpart[u * rowp.nslices + k];
-                mean_row = (double)tot / (double)D;
-                rowp.slot[i] = 0;
+                const double mean_row = (double)tot * inv_D;
+                const float rn = (float)(beta2 * (double)rowp.r[i] + one_minus_beta2 * mean_row);
+                rowp.r[i] = rn;
+                rsum += (double)rn;
             }
-            const float rn = (float)(beta2 * (double)rowp.r[i] + one_minus_beta2 * mean_row);
-            rowp.r[i] = rn;
-            rsum += (double)rn;
+        } else {
+            // sparse step: kRowBatch rows per thread at a time, their map
+            // entries and r loaded together; rows outside the batch's ids
+            // decay, touched rows add their sums of g^2
+            for (int64_t i0 = (int64_t)rb * kStateThreads + threadIdx.x; i0 < V; i0 += stride * kRowBatch) {
+                int sl[kRowBatch];
+                float rr[kRowBatch];
+#pragma unroll
+                for (int k = 0; k < kRowBatch; ++k) {
+                    const int64_t i = i0 + k * stride;
+                    sl[k] = (i < V) ? rowp.slot[i] : 0;
+                    rr[k] = (i < V) ? rowp.r[i] : 0.f;
+                }
+#pragma unroll
+                for (int k = 0; k < kRowBatch; ++k) {
+                    const int64_t i = i0 + k * stride;
+                    if (i >= V)
+                        break;
+                    double mean_row = 0.0;
+                    if (sl[k]) {
+                        const int64_t u = sl[k] - 1;
+                        float tot = 0.f;
+                        for (int q = 0; q < rowp.nslices; ++q)
+                            tot += rowp.rowpart[u * rowp.nslices + q];
+                        mean_row = (double)tot * inv_D;
+                        rowp.slot[i] = 0;
+                    }
+                    const float rn = (float)(beta2 * (double)rr[k] + one_minus_beta2 * mean_row);
+                    rowp.r[i] = rn;
+                    rsum += (double)rn;
+                }
+            }
         }
 #pragma unroll
         for (int o = 16; o >= 1; o >>= 1)
@@ -316,29 +343,42 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
             rsum_part[rb] = t;
         }
     }
-    double csum = 0.0, rsum = 0.0;
     if (threadIdx.x == 0) {
         __threadfence();
         const unsigned t = atomicAdd(&sc->ticket, 1u);
         am_last = (t == gridDim.x - 1);
     }
     __syncthreads();
-    if (am_last && w == 0) {
-        __threadfence();
-        // lane l sums entries l, l + 32, ... in order, then a fixed butterfly
-        for (int b = lane; b < nstate; b += 32)
-            csum += __ldcg(csum_part + b);
-        for (int b = lane; b < nrsum; b += 32)
-            rsum += __ldcg(rsum_part + b);
+    if (!am_last)
+        return;
+    __threadfence();
+    // The last CTA: thread t sums entries t, t + 256, ... in order (all its
+    // loads in flight at once), then a fixed butterfly per warp and the
+    // warps in order.
+    double csum = 0.0, rsum = 0.0;
+    for (int b = threadIdx.x; b < nstate; b += kStateThreads)
+        csum += __ldcg(csum_part + b);
+    for (int b = threadIdx.x; b < nrsum; b += kStateThreads)
+        rsum += __ldcg(rsum_part + b);
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) {
-            csum += __shfl_xor_sync(0xffffffffu, csum, o);
-            rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
-        }
+    for (int o = 16; o >= 1; o >>= 1) {
+        csum += __shfl_xor_sync(0xffffffffu, csum, o);
+        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
     }
-    if (am_last && threadIdx.x == 0) {
-        const double rbar = rsum * inv_bc / (double)V;
-        const double cbar = csum * inv_bc / (double)D;
+    if (lane == 0) {
+        part[w][0] = csum;
+        part[w][1] = rsum;
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        csum = 0.0;
+        rsum = 0.0;
+        for (int q = 0; q < kW; ++q) {
+            csum += part[q][0];
+            rsum += part[q][1];
+        }
+        const double rbar = rsum * inv_bc * inv_V;
+        const double cbar = csum * inv_bc * inv_D;
         const double s = sqrt(rbar * cbar);
         sc->s = s;
         sc->rbar = rbar;

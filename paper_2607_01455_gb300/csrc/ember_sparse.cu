@@ -860,8 +860,8 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
              carry, S, rowpart, colpart, D, NS, nw);
     tr.mark();
     // row pass (all V rows) and column pass in one launch
-    const int64_t vb = (a.V + kStateThreads - 1) / kStateThreads;
-    const int GV = (int)(vb < kMaxRowCtas ? vb : kMaxRowCtas);
+    const int64_t vb = (a.V + (int64_t)kStateThreads * kRowBatch - 1) / ((int64_t)kStateThreads * kRowBatch);
+    const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
     launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
                  a.inv_bc, a.stream, tr.pdl(), a.r, slot, rowpart, NS, GV);
     tr.mark();
