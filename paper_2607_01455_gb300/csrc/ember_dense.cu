@@ -242,9 +242,9 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
 
     if ((int)blockIdx.x < nstate) {
         const int j = blockIdx.x * kStateCols + lane;
-        // rows w, w + 8, w + 16, ...: sixteen loads in flight, summed pairwise
+        // rows w, w + 8, w + 16, ...: 32 loads in flight, summed pairwise
         // in fp32 within the batch and in fp64 across batches
-        constexpr int kBatch = 16;
+        constexpr int kBatch = 32;
         double acc = 0.0;
         if (j < D)
             for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {

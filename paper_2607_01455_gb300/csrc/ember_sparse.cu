@@ -656,7 +656,7 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
 // The update of the touched rows: W[uniq[u]] from the summed row S[u].
 // Three CTAs per SM (two for the widest rows): each CTA has only a few rows,
 // so more of them are kept in flight at once.
-constexpr int apply_ctas_per_sm(int cpt) { return cpt >= 8 ? 2 : 3; }
+constexpr int apply_ctas_per_sm(int cpt) { return cpt >= 8 ? 2 : cpt >= 4 ? 4 : 3; }
 template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, apply_ctas_per_sm(CPT))
 k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__restrict__ rows,
