@@ -67,12 +67,13 @@ def check_dedup(emb, ids):
     np.testing.assert_array_equal(counts.cpu().numpy(), want_c)
 
 
-# 1024-key sort tiles: 4096, 4097, 32768 and 32769 sit on tile edges; the
-# largest batches span 64 tiles.
+# 1024-key sort tiles: 4096, 4097, 32768, 32769, 65536 and 65537 sit on tile
+# edges; the largest batch spans 98 tiles.
 @pytest.mark.parametrize("V,D,N", [
     (50, 8, 1), (50, 8, 37), (1000, 64, 4096), (1000, 64, 4097), (5000, 200, 9000),
     (3000, 203, 5000), (262144, 128, 12288), (100, 2048, 3000), (20000, 8192, 700),
     (262144, 8, 32768), (7, 8, 32768), (70000, 8, 32769), (5000, 8, 65536), (300000, 16, 50000),
+    (5000, 8, 65537), (400000, 8, 100000),
 ])
 @pytest.mark.parametrize("idtype", [torch.int64, torch.int32])
 def test_dedup_bit_exact(cuda_device, V, D, N, idtype):
