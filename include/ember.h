@@ -13,8 +13,7 @@
  *   W_ij <- W_ij - lr * g_ij / (sqrt(rhat_i chat_j / s) + eps)
  *
  * The V x D preconditioner rhat chat^T / s is never stored: it is applied as
- * a per-row and a per-column scaling (Section 2.3, "The preconditioner is
- * never stored").  The sparse step (Section 2.2) takes the token ids of a
+ * a per-row and a per-column scaling, as Section 2.3 prescribes.  The sparse step (Section 2.2) takes the token ids of a
  * batch and one gradient row per occurrence; it equals the dense step on the
  * V x D gradient whose row u is the sum of the rows of every occurrence of u.
  *
@@ -33,8 +32,8 @@
  *     the workspace).
  *   - Results are deterministic: the same inputs give bit-identical W and
  *     state on every run.  No floating-point atomics are used; every sum is
- *     taken in a fixed order (Section 2.3, "deterministic reduction with no
- *     atomic adds").
+ *     taken in a fixed order (the deterministic, atomic-free reduction that
+ *     Section 2.3 asks for).
  */
 #ifndef EMBER_H
 #define EMBER_H

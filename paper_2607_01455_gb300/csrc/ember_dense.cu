@@ -2,8 +2,8 @@
 // Section 2.1) for sm_103a.
 //
 // The step needs two passes over the fp32 gradient G: the update of any
-// element needs chat_j and s, which depend on every row of G (Section 2.3:
-// "The statistics r and c are sums of g^2").  The passes are:
+// element needs chat_j and s, which depend on every row of G (Section 2.3
+// builds both statistics from sums of g^2).  The passes are:
 //
 //   reduce  (k_reduce_dense)  one read of G.  Per row: sum_j g^2, the row EMA
 //           r_i <- beta2 r_i + (1-beta2) mean_j g^2 (Algorithm 1's row second
@@ -26,7 +26,7 @@
 // Determinism: no floating-point atomics.  Every CTA owns a fixed row range
 // (a function of V only), every in-CTA sum has a fixed shape, and the
 // cross-CTA sums run in CTA order, so W and the state are bit-identical
-// from run to run (Section 2.3: "bitwise identical").
+// from run to run, as Section 2.3 requires.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
