@@ -19,8 +19,9 @@
  *
  * Precision and readings (each one is also listed in the design notes):
  *   - all arithmetic is fp64; sums run in plain index order;
- *   - the state vectors r (V floats) and c (D floats) are stored as fp32, which
- *     is how the paper's model-scaling table of Section 3.1 counts them; the rest of the step uses the stored fp32 values;
+ *   - the state vectors r (V floats) and c (D floats) are stored as fp32,
+ *     which is how the paper's model-scaling table of Section 3.1 counts
+ *     them; the rest of the step uses the stored fp32 values;
  *   - the weights are rounded once per step to their storage type (fp32 or
  *     bfloat16) with round-to-nearest-even;
  *   - the paper ascends a reward; this oracle descends a loss by default
