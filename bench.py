@@ -20,6 +20,7 @@ import json
 import os
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -287,10 +288,13 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
+    # where the raw samples go (EMBER_CLOCK_LOG_DIR, default: the temp dir)
+    LOG_DIR = os.environ.get("EMBER_CLOCK_LOG_DIR") or tempfile.gettempdir()
+
     def __init__(self, gpu_index):
         self.gpu_index = gpu_index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_gpu{gpu_index}.csv")
+        self.path = os.path.join(self.LOG_DIR, f"ember_clocks_gpu{gpu_index}.csv")
 
     def __enter__(self):
         try:

@@ -17,7 +17,7 @@
  *   vtil = rhat chat^T / s_t                              factored preconditioner
  *   theta_t = theta_{t-1} -/+ alpha g_t / (sqrt(vtil) + eps)   update
  *
- * Precision and readings (each one is also listed in the design notes):
+ * Precision and readings of the paper:
  *   - all arithmetic is fp64; sums run in plain index order;
  *   - the state vectors r (V floats) and c (D floats) are stored as fp32,
  *     which is how the paper's model-scaling table of Section 3.1 counts

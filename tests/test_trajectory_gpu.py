@@ -11,7 +11,7 @@ bar.  Bounds used (K steps):
   bf16 W:   at most K ulps (one rounding that may land the other way per
             step), and more than 1 ulp on at most 1 % of the elements
   r, c:     relative 1e-5, exact zeros stay exact
-The measured drift is printed (pytest -s) for the design notes.
+The measured drift is printed (pytest -s).
 """
 import numpy as np
 import pytest
