@@ -207,3 +207,33 @@ def test_lmhead_full_size_sampled(cuda_device):
     if bool(far.any()):
         wa, wb = W[far].double(), Wb[far].double()
         assert float(((wa - wb).abs() / wb.abs().clamp(min=wl.lr)).max()) <= 1e-5
+
+
+def test_step_lmhead_graph_capture_matches_eager(cuda_device):
+    """The fused step (cluster launch of the tensor-core kernel, state, apply)
+    is a fixed sequence of launches, so a CUDA graph of it replays to the
+    eager result, bit for bit, and keeps stepping correctly."""
+    V, D, T = 2048, 1024, 300
+    e1, e2 = make(V, D), make(V, D)
+    W0 = (torch.randn(V, D, device=cuda_device) * 0.02).to(torch.bfloat16)
+    W1, W2 = W0.clone(), W0.clone()
+    G1, G2 = torch.empty(V, D, device=cuda_device), torch.empty(V, D, device=cuda_device)
+    dl, h = synth.lmhead_inputs(V, D, T, seed=6, t=1, device=cuda_device)
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        e2.step_lmhead(W2, dl, h, G2, 1e-3, 1, stream=s)  # warm-up on the side stream
+        W2.copy_(W0)
+        e2.state.zero_()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=s):
+        e2.step_lmhead(W2, dl, h, G2, 1e-3, 1, stream=s)
+    for _ in range(2):  # two replays = two steps at t = 1 (the t is baked into the graph)
+        graph.replay()
+        e1.step_lmhead(W1, dl, h, G1, 1e-3, 1)
+    torch.cuda.synchronize()
+    assert e2.device_status() == 0
+    assert torch.equal(G1.view(torch.int32), G2.view(torch.int32))
+    assert torch.equal(W1.view(torch.int16), W2.view(torch.int16))
+    assert torch.equal(e1.state.view(torch.int32), e2.state.view(torch.int32))
