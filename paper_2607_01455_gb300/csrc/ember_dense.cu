@@ -486,12 +486,37 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
 // gradient still in registers: 4VD + 2wVD bytes instead of the full
 // preconditioner's 8VD + 2wVD.  Column sums of g^2 are still accumulated so
 // that c (part of the same V + D state) is maintained by the state pass.
-template <int VEC, int CPT, int R, bool BF16>
+//
+// With ASYNC (16-byte column slices), each thread copies its own elements of
+// the next iteration's rows into shared memory with cp.async while the
+// current rows are reduced and updated, so the two barriers of each
+// iteration no longer leave HBM without requests.  A thread reads back only
+// what it copied itself: the copies need no barrier.
+template <int CPT, int R, bool BF16>
+constexpr size_t rowonly_stage_bytes() { return (size_t)2 * R * CPT * kThreads * (16 + (BF16 ? 8 : 16)); }
+
+__device__ __forceinline__ void cp_async16(void *smem, const void *gmem)
+{
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async8(void *smem, const void *gmem)
+{
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"((uint32_t)__cvta_generic_to_shared(smem)),
+                 "l"(gmem)
+                 : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void cp_async_wait_prev() { asm volatile("cp.async.wait_group 1;" ::: "memory"); }
+
+template <int VEC, int CPT, int R, bool BF16, bool ASYNC>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__restrict__ r,
                 float *__restrict__ colpart, double *__restrict__ rsum_part, int64_t V, int D, int tpr,
                 double beta2, double one_minus_beta2, float inv_bc, float eps, float lr_signed)
 {
+    static_assert(!ASYNC || VEC == 4, "the staged copies move 16-byte slices");
     using F = typename Vec<VEC>::F;
     using WT = typename WRaw<BF16, VEC>::T;
     constexpr int kWarps = kThreads / 32;
@@ -508,8 +533,43 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
     __shared__ float red[kWarps][R];
     __shared__ float rs_sh[kThreads / 32 * R];  // sqrt(rhat) of this iteration's rows
     __shared__ double rsum_sh[kWarps];
+    // ASYNC: two stages of [R][CPT][kThreads] slices of G, then of W; the
+    // column-sum combine buffer (D floats) follows
+    extern __shared__ __align__(16) unsigned char ro_dyn[];
+    constexpr int kWB = BF16 ? 8 : 16;
+    constexpr size_t kStageG = (size_t)2 * R * CPT * kThreads * 16;
+    auto sg_at = [&](int buf, int k, int c) {
+        return ro_dyn + ((size_t)((buf * R + k) * CPT + c) * kThreads + tid) * 16;
+    };
+    auto sw_at = [&](int buf, int k, int c) {
+        return ro_dyn + kStageG + ((size_t)((buf * R + k) * CPT + c) * kThreads + tid) * kWB;
+    };
     grid_dep_wait();
     grid_dep_launch();
+    auto stage = [&](int64_t base, int buf) {  // one commit group per call
+        if constexpr (ASYNC) {
+#pragma unroll
+            for (int k = 0; k < R; ++k) {
+                const int64_t i = base + (int64_t)g * R + k;
+#pragma unroll
+                for (int c = 0; c < CPT; ++c) {
+                    const int col = l + c * tpr;
+                    if (i < row1 && col < DV) {
+                        const int64_t idx = i * D + (int64_t)col * VEC;
+                        cp_async16(sg_at(buf, k, c), G + idx);
+                        if constexpr (BF16)
+                            cp_async8(sw_at(buf, k, c), static_cast<const unsigned short *>(W) + idx);
+                        else
+                            cp_async16(sw_at(buf, k, c), static_cast<const float *>(W) + idx);
+                    }
+                }
+            }
+            cp_async_commit();
+        }
+    };
+    int buf = 0;
+    if (ASYNC && row0 < row1)
+        stage(row0, 0);
 
     float acc[CPT][VEC];
 #pragma unroll
@@ -522,6 +582,14 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
     for (int64_t base = row0; base < row1; base += rows_per_it) {
         F v[R][CPT];
         WT wr[R][CPT];
+        if constexpr (ASYNC) {
+            // the next iteration's copies go out, this one's have landed
+            if (base + rows_per_it < row1)
+                stage(base + rows_per_it, buf ^ 1);
+            else
+                cp_async_commit();
+            cp_async_wait_prev();
+        }
 #pragma unroll
         for (int k = 0; k < R; ++k) {
             const int64_t i = base + (int64_t)g * R + k;
@@ -529,11 +597,18 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
             for (int c = 0; c < CPT; ++c) {
                 const int col = l + c * tpr;
                 const bool in = i < row1 && col < DV;
-                v[k][c] = in ? load_g<VEC>(G + i * D + (int64_t)col * VEC) : zero_vec<VEC>();
-                if (in)
-                    wr[k][c] = load_w<BF16, VEC>(W, i * D + (int64_t)col * VEC);
+                if constexpr (ASYNC) {
+                    v[k][c] = in ? *reinterpret_cast<const F *>(sg_at(buf, k, c)) : zero_vec<VEC>();
+                    if (in)
+                        wr[k][c] = *reinterpret_cast<const WT *>(sw_at(buf, k, c));
+                } else {
+                    v[k][c] = in ? load_g<VEC>(G + i * D + (int64_t)col * VEC) : zero_vec<VEC>();
+                    if (in)
+                        wr[k][c] = load_w<BF16, VEC>(W, i * D + (int64_t)col * VEC);
+                }
             }
         }
+        buf ^= 1;
         float rp[R];
 #pragma unroll
         for (int k = 0; k < R; ++k) {
@@ -602,7 +677,7 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
                     out[col * VEC + e] = acc[c][e];
         }
     } else {
-        extern __shared__ float colsh[];  // D floats
+        float *colsh = reinterpret_cast<float *>(ro_dyn + (ASYNC ? rowonly_stage_bytes<CPT, R, BF16>() : 0));
         for (int q = 0; q < rg; ++q) {
             if (g == q) {
 #pragma unroll
@@ -712,16 +787,26 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     if (a.variant == EMBER_VARIANT_ROW && !a.lm) {
         // one pass over G and W, then the column state; no apply pass
         constexpr int RR = (4 / CPT) < 1 ? 1 : (4 / CPT);
+        constexpr bool kAsync = VEC == 4;
         if (a.trace)
             cudaEventRecord(a.trace[0], a.stream);
-        if (a.wbf16)
-            e = launch_k(k_rowonly_dense<VEC, CPT, RR, true>, dim3(nparts), dim3(kThreads), shmem, a.stream,
-                         false, a.W, a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2,
-                         a.one_minus_beta2, (float)a.inv_bc, a.eps, a.lr_signed);
-        else
-            e = launch_k(k_rowonly_dense<VEC, CPT, RR, false>, dim3(nparts), dim3(kThreads), shmem, a.stream,
-                         false, a.W, a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2,
-                         a.one_minus_beta2, (float)a.inv_bc, a.eps, a.lr_signed);
+        if (a.wbf16) {
+            auto *k = k_rowonly_dense<VEC, CPT, RR, true, kAsync>;
+            const size_t sm = shmem + (kAsync ? rowonly_stage_bytes<CPT, RR, true>() : 0);
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e == cudaSuccess)
+                e = launch_k(k, dim3(nparts), dim3(kThreads), sm, a.stream, false, a.W, a.G, a.r, colpart,
+                             rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, (float)a.inv_bc, a.eps,
+                             a.lr_signed);
+        } else {
+            auto *k = k_rowonly_dense<VEC, CPT, RR, false, kAsync>;
+            const size_t sm = shmem + (kAsync ? rowonly_stage_bytes<CPT, RR, false>() : 0);
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e == cudaSuccess)
+                e = launch_k(k, dim3(nparts), dim3(kThreads), sm, a.stream, false, a.W, a.G, a.r, colpart,
+                             rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, (float)a.inv_bc, a.eps,
+                             a.lr_signed);
+        }
         if (e != cudaSuccess)
             return e;
         if (a.trace)
