@@ -27,6 +27,15 @@
 // (a function of V only), every in-CTA sum has a fixed shape, and the
 // cross-CTA sums run in CTA order, so W and the state are bit-identical
 // from run to run, as Section 2.3 requires.
+//
+// The same launcher also runs:
+//   - the row-only variant in one pass (k_rowonly_dense), no apply pass;
+//   - the LM-head step: the tensor-core kernel of ember_lmhead.cu forms G and
+//     its per-tile sums of g^2, the state pass finishes them (row pass from
+//     per-column-block sums), then the apply pass;
+//   - the two phases of a row-sharded step: the reduce pass or the apply
+//     pass over one shard's CTAs of the whole-table grid (RowSpan), and the
+//     state pass on every shard's gathered partials.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>

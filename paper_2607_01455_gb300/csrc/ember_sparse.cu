@@ -23,7 +23,8 @@
 //             a touched row to its distinct-id index.
 //   segsum    k_sp_segsum, k_sp_carry: the summed gradient row of every
 //             distinct id, adding its occurrences in increasing occurrence
-//             order; per (id, column slice) sums of g^2; per-CTA column sums
+//             order (compensated fp32 sums); per (id, column slice) sums of
+//             g^2; per-CTA column sums
 //             of g^2.  Each worker owns a contiguous, equal share of the
 //             sorted occurrences, so the work is even however skewed the id
 //             counts are (a Zipf head id can own thousands of occurrences);
