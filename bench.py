@@ -32,11 +32,11 @@ NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of the apply kernel
-# on the default workload (V=128256, D=8192, bf16 W), from the one-pass ncu
+# dram__bytes_read.sum + dram__bytes_write.sum per launch of the apply kernel,
+# by workload (V=128256, D=8192, bf16 W: the default), from the one-pass ncu
 # capture summarised in profiles/dense_lmhead_v128256_d8192_bf16_launches.md.
 # Set to None whenever k_apply_dense changes until it is captured again.
-APPLY_TRAFFIC_BYTES = 8374837546
+APPLY_TRAFFIC_BYTES = {"dense_lmhead_v128256_d8192_bf16": None}
 # The same for k_lmhead_grad on the LM-head gradient workload (V=128256,
 # D=8192, T=4096), from profiles/lmhead_grad_v128256_d8192_t4096_bf16_launches.md.
 # Set to None whenever k_lmhead_grad changes until it is captured again.
@@ -53,6 +53,17 @@ def step_bytes(wl):
     state read and written once."""
     V, D, w = wl.V, wl.D, wbytes(wl)
     return (8 + 2 * w) * V * D + 8 * (V + D)
+
+
+def column_panels(D):
+    """Column panels the library splits a D-wide table into: a CTA holds
+    8192 columns of a row with 16-byte accesses (D % 4 == 0), 2048 without;
+    wider tables run in equal panels, one reduce and one apply launch each."""
+    vec = 4 if D % 4 == 0 else 1
+    maxw = 2048 * vec
+    n = -(-D // maxw)
+    pw = -(-(-(-D // n)) // vec) * vec
+    return -(-D // pw)
 
 
 def kernel_bytes(wl):
@@ -170,8 +181,13 @@ def run_row_only(wl, dev, steps, warmup, flush, W, G):
         raise SystemExit("device status after the row-only steps")
     ms = sum(a.elapsed_time(b) for a, b in ev) / steps
     B = (4 + 2 * wbytes(wl)) * wl.V * wl.D + 8 * (wl.V + wl.D)
+    npan = column_panels(wl.D)
+    # a table in column panels has no one-pass kernel: reduce, state and
+    # apply passes per step, G read twice
+    launches = 2 if npan == 1 else 2 * npan + 1
     return {"variant": "row", "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
-            "algorithmic_bytes": B, "params_per_s": wl.V * wl.D / (ms * 1e-3), "gpu_launches": 2 * steps}
+            "algorithmic_bytes": B, "params_per_s": wl.V * wl.D / (ms * 1e-3), "gpu_launches": launches * steps,
+            "one_pass": npan == 1}
 
 
 LMHEAD_KERNELS = ["lmhead_grad", "state", "apply"]
@@ -505,6 +521,7 @@ def run_ours(args, world, rank, local):
     G = synth.dense_grad(wl, rank, 1, dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
+    npan = column_panels(wl.D)
 
     def one_step(t, ev):
         emb.trace(ev)
@@ -563,9 +580,12 @@ def run_ours(args, world, rank, local):
     roofline = {
         "bound": "hbm", "kernel": "k_apply_dense", "achieved": kern[dom]["gbs"], "peak": peak,
         "unit": "GB/s", "frac": kern[dom]["gbs"] / peak, "peak_kind": peak_kind,
-        "traffic": APPLY_TRAFFIC_BYTES,
+        "traffic": APPLY_TRAFFIC_BYTES.get(wl.name),
         "algorithmic_bytes_per_launch": kb[dom],
     }
+    if npan > 1:
+        # one apply launch per column panel: the figures are per pass
+        roofline["launches_per_pass"] = npan
 
     # end to end through the C ABI: the gradient comes in from pinned host
     # memory, the step runs, and its result -- the optimizer state r, c
@@ -650,7 +670,7 @@ def run_ours(args, world, rank, local):
         "roofline": roofline,
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": (2 * npan + 1) * args.steps,
         "clocks": clocks.summary(),
         "params_per_s": world * wl.V * wl.D / (ms * 1e-3),
         "frac_of_nominal_8TBs": value / world / NOMINAL_HBM_GBS,

@@ -90,8 +90,15 @@ void ember_hparams_default(ember_hparams *hp);
 
 /* Create a host-side handle for one V x D table whose weights are stored as
  * wdtype.  hp == NULL takes the defaults.  Validates V >= 1, D >= 1,
- * V * D < 2^62, 0 <= beta2 < 1, eps >= 0 (finite) and the enums.  Touches no
- * GPU.  On success *out owns a handle to free with ember_destroy(). */
+ * V * D < 2^62, 0 <= beta2 < 1, eps >= 0 (finite) and the enums
+ * (EMBER_ERR_INVALID_ARG), and V < 2^31, D <= 65536 (EMBER_ERR_UNSUPPORTED).
+ * Touches no GPU.  On success *out owns a handle to free with
+ * ember_destroy().
+ *   Tables whose rows a CTA cannot hold whole (D > 8192 on the 16-byte
+ * vector path, D > 2048 on the scalar one) are processed in column panels
+ * of equal width: one reduce and one apply launch per panel, each row's sum
+ * of g^2 added up from per-panel partial sums in panel order.  Every step
+ * accepts them except the row-sharded one and ember_step_dense_noalloc. */
 ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp,
                           ember_wdtype wdtype, ember_handle **out);
 
@@ -155,8 +162,9 @@ ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G
  * no workspace is bound or used: the scratch (column and row-sum partials,
  * scalars) lives in a 10 MiB array inside the library, present on every GPU
  * that loads the library until the process exits.  Nothing is allocated.
- * Every table this library accepts fits (D <= 8192 needs 9.97 MB); a larger
- * need returns EMBER_ERR_WORKSPACE.
+ * Every table whose rows a CTA holds whole fits (D <= 8192 needs 9.97 MB);
+ * a table processed in column panels (see ember_create) returns
+ * EMBER_ERR_WORKSPACE.
  *   The first call on each device looks up the array's device address
  * (cudaGetSymbolAddress) with that device current; make that first call
  * before any stream capture.  All calls on a device share the one array and
@@ -233,7 +241,9 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
  *   block: ember_shard_exchange_bytes(h, nshards) bytes, device, 256-byte
  *       aligned; blocks: nshards of them back to back, in shard order.
  * Variant ROW is not offered (EMBER_ERR_UNSUPPORTED): its one-pass kernel
- * needs no exchange for W and is run per shard with ember_step_dense. */
+ * needs no exchange for W and is run per shard with ember_step_dense.  Nor
+ * are tables processed in column panels (see ember_create;
+ * EMBER_ERR_UNSUPPORTED). */
 int64_t ember_shard_rows(const ember_handle *h, int shard, int nshards, int64_t *row0);
 size_t ember_shard_exchange_bytes(const ember_handle *h, int nshards);
 ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const float *G_shard, float *state,

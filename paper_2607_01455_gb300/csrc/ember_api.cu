@@ -394,6 +394,8 @@ static ember_status shard_common(ember_handle *h, int shard, int nshards, const 
     a->trace = nullptr;
     if (!choose_colmap(h->D, vec4, &a->map))
         return EMBER_ERR_UNSUPPORTED;
+    if (a->map.npanels != 1)
+        return EMBER_ERR_UNSUPPORTED;  // a shard's rows must fit one CTA whole
     return EMBER_OK;
 }
 

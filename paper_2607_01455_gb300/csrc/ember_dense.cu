@@ -53,12 +53,15 @@ using namespace dev;
 // STAGE: G is read from host memory the GPU can address (over the
 // Grace-Blackwell chip-to-chip link) and every element is also written to
 // G_stage in HBM for the apply pass.
+// D is the number of columns this launch covers and ld the row stride of G
+// and colpart: a column panel of a wider table has D < ld, and then each
+// row's sum of g^2 over the panel goes to rowpart[i] instead of into r.
 template <int VEC, int CPT, int R, bool STAGE>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                float *__restrict__ colpart, double *__restrict__ rsum_part,
-               int64_t V, int D, int tpr, double beta2, double one_minus_beta2,
-               float *__restrict__ G_stage, RowSpan span)
+               int64_t V, int D, int ld, int tpr, double beta2, double one_minus_beta2,
+               float *__restrict__ G_stage, float *__restrict__ rowpart, RowSpan span)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
@@ -103,12 +106,12 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                 const int col = l + c * tpr;
                 const bool in = i < row1 && col < DV;
                 if constexpr (STAGE) {
-                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
+                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
                     v[k][c] = in ? *reinterpret_cast<const F *>(G + idx) : zero_vec<VEC>();
                     if (in)
                         *reinterpret_cast<F *>(G_stage + idx) = v[k][c];
                 } else {
-                    v[k][c] = in ? load_g<VEC>(G + (i - span.row_base) * D + (int64_t)col * VEC)
+                    v[k][c] = in ? load_g<VEC>(G + (i - span.row_base) * ld + (int64_t)col * VEC)
                                  : zero_vec<VEC>();
                 }
             }
@@ -161,6 +164,10 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                     float sum = 0.f;
                     for (int k = 0; k < wpg; ++k)
                         sum += red[gq * wpg + k][q];
+                    if (rowpart) {
+                        rowpart[i] = sum;
+                        continue;
+                    }
                     const double mean_row = (double)sum / (double)D;
                     const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
                     r[i] = rn;
@@ -174,7 +181,7 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     }
 
     // column partial of this CTA: row groups combined in order 0 .. rg-1
-    float *out = colpart + (int64_t)blockIdx.x * D;
+    float *out = colpart + (int64_t)blockIdx.x * ld;
     if (rg == 1) {
 #pragma unroll
         for (int c = 0; c < CPT; ++c) {
@@ -210,7 +217,7 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     if (lane == 0)
         rsum_sh[warp] = rsum;
     __syncthreads();
-    if (tid == 0) {
+    if (tid == 0 && rowpart == nullptr) {
         double s = 0.0;
         for (int q = 0; q < kWarps; ++q)
             s += rsum_sh[q];
@@ -399,12 +406,13 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
 
 // Pass 3: the update.  Same row ranges and column mapping as pass 1; each
 // CTA walks its rows from the last iteration block to the first.  The
-// column scales live in shared memory (D floats).
+// column scales live in shared memory (D floats).  D columns from row stride
+// ld, as in pass 1: W, G and c point at the first column of the panel.
 template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__restrict__ r,
               const float *__restrict__ c, const DevScalars *__restrict__ sc,
-              int64_t V, int D, int tpr, float inv_bc, float eps, float lr_signed, int variant,
+              int64_t V, int D, int ld, int tpr, float inv_bc, float eps, float lr_signed, int variant,
               RowSpan span)
 {
     using F = typename Vec<VEC>::F;
@@ -429,7 +437,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (i < row1 && col < DV) {
-                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
+                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
                     asm volatile("prefetch.global.L2 [%0];" ::"l"(G + idx));
                     asm volatile("prefetch.global.L2 [%0];" ::"l"(static_cast<const char *>(W) +
                                                                    idx * (BF16 ? 2 : 4)));
@@ -457,7 +465,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (i < row1 && col < DV) {
-                    const int64_t idx = (i - span.row_base) * D + (int64_t)col * VEC;
+                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
                     gv[k][cc] = load_g<VEC>(G + idx);
                     wr[k][cc] = load_w<BF16, VEC>(W, idx);
                 }
@@ -482,7 +490,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
                     const float u = comp(gv[k][cc], e) / den;
                     w[e] = fmaf(lr_signed, u, w[e]);
                 }
-                store_w<BF16, VEC>(W, (i - span.row_base) * D + (int64_t)col * VEC, w);
+                store_w<BF16, VEC>(W, (i - span.row_base) * ld + (int64_t)col * VEC, w);
             }
         }
     }
@@ -750,7 +758,13 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     double *csum_part = reinterpret_cast<double *>(a.ws + a.lay.csum_part);
     float *colpart = reinterpret_cast<float *>(a.ws + a.lay.colpart);
     const int rg = kThreads / a.map.tpr;
-    const size_t shmem = (rg > 1) ? (size_t)D * sizeof(float) : 0;
+    // column panels (one unless D is wider than a CTA's row): columns
+    // [q pw, q pw + cols(q)) with row stride D
+    const int np = a.map.npanels;
+    const int pw = a.map.pw;
+    const int ld = (int)a.D;
+    auto cols = [&](int q) { return (q + 1 < np) ? pw : (int)(a.D - (int64_t)q * pw); };
+    const size_t shmem = (rg > 1) ? (size_t)pw * sizeof(float) : 0;
 
     // With tracing, events sit between the kernels and each launch simply
     // follows the previous one; without, kernels 2 and 3 use programmatic
@@ -762,6 +776,8 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         // one phase of a row-sharded step: the shard's own CTAs of the
         // whole-table grid, so each per-CTA partial equals the unsharded one
         const ShardArgs &sh = *a.shard;
+        if (np != 1)
+            return cudaErrorInvalidValue;  // refused by the entry points
         const int ncta = sh.cta_end - sh.cta_begin;
         span = RowSpan{sh.cta_begin, nparts, sh.row_base};
         if (sh.phase == 1) {
@@ -770,7 +786,8 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             float *bcol = static_cast<float *>(sh.block);
             double *brsum = reinterpret_cast<double *>(static_cast<unsigned char *>(sh.block) + sh.block_rsum);
             e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(ncta), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, bcol, brsum, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr, span);
+                         a.G, a.r, bcol, brsum, a.V, D, ld, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr,
+                         nullptr, span);
             return e != cudaSuccess ? e : cudaGetLastError();
         }
         e = launch_k(k_shard_unpack, dim3(kGridCtas), dim3(kThreads), 0, a.stream, false,
@@ -785,15 +802,15 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         const size_t cs_bytes = (size_t)D * sizeof(float);
         if (a.wbf16)
             e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
-                         a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
                          a.variant, span);
         else
             e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
-                         a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
                          a.variant, span);
         return e != cudaSuccess ? e : cudaGetLastError();
     }
-    if (a.variant == EMBER_VARIANT_ROW && !a.lm) {
+    if (a.variant == EMBER_VARIANT_ROW && !a.lm && np == 1) {
         // one pass over G and W, then the column state; no apply pass
         constexpr int RR = (4 / CPT) < 1 ? 1 : (4 / CPT);
         constexpr bool kAsync = VEC == 4;
@@ -853,38 +870,60 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         if (e != cudaSuccess)
             return e;
     } else {
+        // with several column panels each reduce launch leaves its rows' sums
+        // of g^2 over the panel in rowpart[q][V] (the LM-head step's region),
+        // and the state pass adds them up per row in panel order
+        float *rowpart = (np > 1) ? reinterpret_cast<float *>(a.ws + a.lay.lm_rowpart) : nullptr;
         if (a.trace)
             cudaEventRecord(a.trace[0], a.stream);
-        if (a.G_stage)
-            e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, a.G_stage, span);
-        else
-            e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, colpart, rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr, span);
-        if (e != cudaSuccess)
-            return e;
+        for (int q = 0; q < np; ++q) {
+            const int64_t c0 = (int64_t)q * pw;
+            float *rp = rowpart ? rowpart + (int64_t)q * a.V : nullptr;
+            if (a.G_stage)
+                e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream,
+                             pdl && q > 0, a.G + c0, a.r, colpart + c0, rsum_part, a.V, cols(q), ld, a.map.tpr,
+                             a.beta2, a.one_minus_beta2, a.G_stage + c0, rp, span);
+            else
+                e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream,
+                             pdl && q > 0, a.G + c0, a.r, colpart + c0, rsum_part, a.V, cols(q), ld, a.map.tpr,
+                             a.beta2, a.one_minus_beta2, nullptr, rp, span);
+            if (e != cudaSuccess)
+                return e;
+        }
         if (a.trace)
             cudaEventRecord(a.trace[1], a.stream);
-        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        if (np == 1) {
+            e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
+                             a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        } else {
+            const int64_t vb = (a.V + kStateThreads - 1) / kStateThreads;
+            const int nrow_ctas = (int)(vb < kMaxRowCtas ? vb : kMaxRowCtas);
+            e = launch_state(colpart, nparts, rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D, a.beta2,
+                             a.one_minus_beta2, a.inv_bc, a.stream, pdl, a.r, nullptr, rowpart, np, nrow_ctas);
+        }
         if (e != cudaSuccess)
             return e;
     }
-    // the apply pass reads the staged copy, or the G the LM-head kernel wrote
+    // the apply pass reads the staged copy, or the G the LM-head kernel wrote;
+    // panels from the last (the reduce pass's last rows, still in L2)
     const float *Gd = a.lm ? a.lm->G : a.G_stage ? a.G_stage : a.G;
     if (a.trace)
         cudaEventRecord(a.trace[2], a.stream);
-    const size_t cs_bytes = (size_t)D * sizeof(float);
-    if (a.wbf16)
-        e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
-                     a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
-                     a.eps, a.lr_signed, a.variant, span);
-    else
-        e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
-                     a.stream, pdl, a.W, Gd, a.r, a.c, sc, a.V, D, a.map.tpr, (float)a.inv_bc,
-                     a.eps, a.lr_signed, a.variant, span);
-    if (e != cudaSuccess)
-        return e;
+    const size_t cs_bytes = (size_t)pw * sizeof(float);
+    for (int q = np - 1; q >= 0; --q) {
+        const int64_t c0 = (int64_t)q * pw;
+        void *Wq = static_cast<unsigned char *>(a.W) + c0 * (a.wbf16 ? 2 : 4);
+        if (a.wbf16)
+            e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
+                         a.stream, pdl, Wq, Gd + c0, a.r, a.c + c0, sc, a.V, cols(q), ld, a.map.tpr,
+                         (float)a.inv_bc, a.eps, a.lr_signed, a.variant, span);
+        else
+            e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
+                         a.stream, pdl, Wq, Gd + c0, a.r, a.c + c0, sc, a.V, cols(q), ld, a.map.tpr,
+                         (float)a.inv_bc, a.eps, a.lr_signed, a.variant, span);
+        if (e != cudaSuccess)
+            return e;
+    }
     if (a.trace)
         cudaEventRecord(a.trace[3], a.stream);
     return cudaGetLastError();
@@ -905,8 +944,16 @@ cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, in
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)
 {
+    if (D < 1 || D > kMaxCols)
+        return false;
     const int vec = (vec4_ok && D % 4 == 0) ? 4 : 1;
-    const int64_t DV = D / vec;
+    // equal panels of at most kThreads * 8 accesses, widths a multiple of vec
+    const int64_t maxw = (int64_t)kThreads * 8 * vec;
+    const int64_t np = (D + maxw - 1) / maxw;
+    const int64_t pw = ((D + np - 1) / np + vec - 1) / vec * vec;
+    m->npanels = (int)((D + pw - 1) / pw);
+    m->pw = (int)pw;
+    const int64_t DV = pw / vec;
     for (int tpr = 32; tpr <= kThreads; tpr *= 2) {
         const int64_t need = (DV + tpr - 1) / tpr;
         if (need <= 4 || tpr == kThreads) {

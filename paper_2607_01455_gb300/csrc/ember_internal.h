@@ -88,10 +88,18 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N);
 
 // Column mapping of a V x D row-major table onto the CTA: `vec` consecutive
 // columns per access, `tpr` threads per row, `cpt` accesses per thread per row.
+// A CTA holds kThreads x 8 accesses of one row: 8192 columns with 16-byte
+// accesses, 2048 with 4-byte ones.  Wider tables are split into column
+// panels of equal width (the last one may be narrower), each run as a
+// table of `pw` columns with row stride D; the row sums of g^2 then come
+// from per-panel partial sums.  kMaxCols bounds D.
+constexpr int kMaxCols = 65536;
 struct ColMap {
-    int vec;   // 4 (16-byte fp32 accesses) or 1
-    int tpr;   // threads per row: 32 .. kThreads, a power of two
-    int cpt;   // accesses per thread per row: 1, 2, 4 or 8
+    int vec;      // 4 (16-byte fp32 accesses) or 1
+    int tpr;      // threads per row: 32 .. kThreads, a power of two
+    int cpt;      // accesses per thread per row: 1, 2, 4 or 8
+    int npanels;  // column panels: 1 when a CTA holds a whole row
+    int pw;       // panel width in columns (a multiple of vec); D when npanels == 1
 };
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m);

@@ -14,8 +14,9 @@
 // library call.
 //
 // The array is kNoAllocScratchBytes (10 MiB) on every GPU that loads the
-// library, held until the process exits.  That covers every table width the
-// dense step supports (D <= 8192 needs 9.97 MB); a larger need is refused.
+// library, held until the process exits.  That covers every table a CTA
+// holds whole rows of (D <= 8192 needs 9.97 MB); wider tables, which run in
+// column panels with per-row partial sums, are refused.
 //
 // In host code the array's name is only a host-side stand-in; the kernels get
 // its device address, looked up once per device with cudaGetSymbolAddress on
@@ -76,6 +77,14 @@ extern "C" ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const
     if (need > kNoAllocScratchBytes)
         return EMBER_ERR_WORKSPACE;
 
+    // a table split into column panels also needs per-row partial sums
+    const bool vec4 = (h->D % 4 == 0) && aligned(W, 4 * wsz) && aligned(G, 16);
+    ColMap map;
+    if (!choose_colmap(h->D, vec4, &map))
+        return EMBER_ERR_UNSUPPORTED;
+    if (map.npanels != 1)
+        return EMBER_ERR_WORKSPACE;
+
     unsigned char *scratch = scratch_for_current_device();
     if (!scratch)
         return EMBER_ERR_CUDA;
@@ -102,8 +111,6 @@ extern "C" ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const
     a.lay = lay;
     a.stream = s;
     a.trace = nullptr;
-    const bool vec4 = (h->D % 4 == 0) && aligned(W, 4 * wsz) && aligned(G, 16);
-    if (!choose_colmap(h->D, vec4, &a.map))
-        return EMBER_ERR_UNSUPPORTED;
+    a.map = map;
     return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
 }

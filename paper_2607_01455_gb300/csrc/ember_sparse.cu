@@ -656,14 +656,16 @@ k_sp_carry(const int32_t *__restrict__ segidx, const int32_t *__restrict__ segof
 
 // The update of the touched rows: W[uniq[u]] from the summed row S[u].
 // Three CTAs per SM (two for the widest rows): each CTA has only a few rows,
-// so more of them are kept in flight at once.
+// so more of them are kept in flight at once.  D columns from row stride ld
+// (a column panel of a wider table: W, S, rows and c point at its first
+// column).
 constexpr int apply_ctas_per_sm(int cpt) { return cpt >= 8 ? 2 : cpt >= 4 ? 4 : 3; }
 template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, apply_ctas_per_sm(CPT))
 k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__restrict__ rows,
            const int32_t *__restrict__ uniq, const int32_t *__restrict__ single,
            const float *__restrict__ r, const float *__restrict__ c,
-           const DevScalars *__restrict__ sc, int D, int tpr, float inv_bc, float eps,
+           const DevScalars *__restrict__ sc, int D, int ld, int tpr, float inv_bc, float eps,
            float lr_signed, int variant)
 {
     using F = typename Vec<VEC>::F;
@@ -701,13 +703,13 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
         for (int k = 0; k < R; ++k) {
             const int64_t u = ub + k;
             row[k] = next[k];
-            const float *src = (nsingle[k] >= 0) ? rows + (int64_t)nsingle[k] * D : S + u * D;
+            const float *src = (nsingle[k] >= 0) ? rows + (int64_t)nsingle[k] * ld : S + u * ld;
 #pragma unroll
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (row[k] >= 0 && col < DV) {
                     gv[k][cc] = load_g<VEC>(src + (int64_t)col * VEC);
-                    wr[k][cc] = load_w<BF16, VEC>(W, row[k] * D + (int64_t)col * VEC);
+                    wr[k][cc] = load_w<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC);
                 }
             }
         }
@@ -735,7 +737,7 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
                     const float u = comp(gv[k][cc], e) / den;
                     wv[e] = fmaf(lr_signed, u, wv[e]);
                 }
-                store_w<BF16, VEC>(W, row[k] * D + (int64_t)col * VEC, wv);
+                store_w<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC, wv);
             }
         }
     }
@@ -866,16 +868,24 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
                  a.inv_bc, a.stream, tr.pdl(), a.r, slot, rowpart, NS, GV);
     tr.mark();
-    const size_t cs_bytes = (size_t)D * sizeof(float);
+    // one launch per column panel (one unless D is wider than a CTA's row)
+    const int np = a.map.npanels, pw = a.map.pw;
+    const size_t cs_bytes = (size_t)pw * sizeof(float);
     const int GA = kSms * apply_ctas_per_sm(CPT);
-    if (a.wbf16)
-        launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
-                 S, a.rows, uniq, single, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
-                 a.variant);
-    else
-        launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), a.W,
-                 S, a.rows, uniq, single, a.r, a.c, sc, D, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
-                 a.variant);
+    for (int q = 0; q < np; ++q) {
+        const int64_t c0 = (int64_t)q * pw;
+        const int dq = (q + 1 < np) ? pw : (int)(a.D - c0);
+        void *Wq = static_cast<unsigned char *>(a.W) + c0 * (a.wbf16 ? 2 : 4);
+        const float *rq = a.rows ? a.rows + c0 : nullptr;
+        if (a.wbf16)
+            launch_k(k_sp_apply<VEC, CPT, R, true>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), Wq,
+                     S + c0, rq, uniq, single, a.r, a.c + c0, sc, dq, (int)a.D, a.map.tpr, (float)a.inv_bc, a.eps,
+                     a.lr_signed, a.variant);
+        else
+            launch_k(k_sp_apply<VEC, CPT, R, false>, dim3(GA), dim3(kThreads), cs_bytes, a.stream, tr.pdl(), Wq,
+                     S + c0, rq, uniq, single, a.r, a.c + c0, sc, dq, (int)a.D, a.map.tpr, (float)a.inv_bc, a.eps,
+                     a.lr_signed, a.variant);
+    }
     tr.mark();
     return cudaGetLastError();
 }

@@ -71,11 +71,15 @@ WORKLOADS = {
                  T=4096),
         # a quarter of the head's rows: the size the detailed profiles use
         Workload("lmhead_grad_v32768_d8192_t4096_bf16", 32768, 8192, "bf16", 20, kind="lmhead", T=4096),
+        # an LM head wider than one CTA's row (a 128256-token vocabulary at
+        # hidden size 16384): the step runs in two column panels
+        Workload("dense_wide_v128256_d16384_bf16", 128256, 16384, "bf16", 20, heavy_frac=0.01),
     ]
 }
 # The five workloads of the optimizer step in the order they are listed for
-# the paper's method; the LM-head gradient workload comes after them.
-ORDER = [n for n, w in WORKLOADS.items() if w.kind != "lmhead"]
+# the paper's method; the LM-head gradient and wide-table workloads come
+# after them.
+ORDER = [n for n, w in WORKLOADS.items() if w.kind != "lmhead" and not n.startswith("dense_wide")]
 LOGIT_STD = 2.0
 
 

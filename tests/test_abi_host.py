@@ -87,8 +87,9 @@ def test_paper_state_sizes_through_the_library():
     (dict(V=4, D=4, eps=float("inf")), E.EMBER_ERR_INVALID_ARG),
     (dict(V=4, D=4, variant=3), E.EMBER_ERR_INVALID_ARG),
     (dict(V=4, D=4, maximize=2), E.EMBER_ERR_INVALID_ARG),
-    (dict(V=4, D=8196), E.EMBER_ERR_UNSUPPORTED),
-    (dict(V=4, D=2049), E.EMBER_ERR_UNSUPPORTED),
+    (dict(V=4, D=65537), E.EMBER_ERR_UNSUPPORTED),
+    (dict(V=4, D=1 << 20), E.EMBER_ERR_UNSUPPORTED),
+    (dict(V=1 << 31, D=4), E.EMBER_ERR_UNSUPPORTED),
 ])
 def test_create_rejects(kw, status):
     hp = E.ember_hparams_default()
@@ -125,7 +126,9 @@ def test_lmhead_needs_multiples_of_8(V, D):
 
 
 def test_create_accepts_limits():
-    for V, D in [(1, 8192), (3, 2048), (2, 2047), (1, 3)]:
+    # widths past one CTA's row (8192, or 2048 without 16-byte vectors) run
+    # in column panels, up to 65536
+    for V, D in [(1, 8192), (3, 2048), (2, 2047), (1, 3), (2, 8196), (2, 2049), (1, 65536), (1, 65533)]:
         E.ember_destroy(E.ember_create(V, D))
 
 

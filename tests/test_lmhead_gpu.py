@@ -112,7 +112,7 @@ def test_step_lmhead_gated(cuda_device, V, D, T, wdtype):
         st = emb.state.cpu().numpy()
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
-        check_weights(w_to_host(W), Wo, 1e-3)
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0)
 
 
 @pytest.mark.parametrize("opt", [Opt(variant="row"), Opt(variant="col"), Opt(maximize=True),

@@ -51,7 +51,7 @@ def gated_sparse_step(emb, W, ids, rows, lr, t, opt):
     check_state(st[:V], r, "r")
     check_state(st[V:], c, "c")
     Wg = w_to_host(W)
-    check_weights(Wg, Wo, lr)
+    check_weights(Wg, Wo, lr, prev=W0)
     # rows whose id does not occur keep their weights bit for bit
     touched = np.zeros(V, bool)
     ids_h = ids.cpu().numpy().astype(np.int64)
