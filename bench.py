@@ -36,7 +36,7 @@ L2_FLUSH_BYTES = 512 << 20
 # by workload (V=128256, D=8192, bf16 W: the default), from the one-pass ncu
 # capture summarised in profiles/dense_lmhead_v128256_d8192_bf16_launches.md.
 # Set to None whenever k_apply_dense changes until it is captured again.
-APPLY_TRAFFIC_BYTES = {"dense_lmhead_v128256_d8192_bf16": None}
+APPLY_TRAFFIC_BYTES = {"dense_lmhead_v128256_d8192_bf16": 8374828715}
 # The same for k_lmhead_grad on the LM-head gradient workload (V=128256,
 # D=8192, T=4096), from profiles/lmhead_grad_v128256_d8192_t4096_bf16_launches.md.
 # Set to None whenever k_lmhead_grad changes until it is captured again.
