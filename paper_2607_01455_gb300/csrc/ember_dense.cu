@@ -36,6 +36,10 @@
 //   - the two phases of a row-sharded step: the reduce pass or the apply
 //     pass over one shard's CTAs of the whole-table grid (RowSpan), and the
 //     state pass on every shard's gathered partials.
+//   - tables wider than a CTA holds (more than 8192 columns, or 2048 without
+//     16-byte accesses): the reduce and apply passes once per column panel
+//     with the row stride D, the rows' sums of g^2 per panel added up by the
+//     state pass, in panel order.
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>

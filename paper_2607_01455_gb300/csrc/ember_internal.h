@@ -26,8 +26,9 @@ constexpr int kPartRows = kSparseCtas > kGridCtas ? kSparseCtas : kGridCtas;
 
 // The state pass reduces 32 columns per CTA.  Its row pass runs up to
 // kMaxRowCtas CTAs: about one row per thread for the LM-head step (whose
-// rows each sum ceil(D/256) slices), and kRowBatch rows per thread for the
-// sparse step (whose untouched rows only decay).
+// rows each sum ceil(D/256) slices) and for a dense step in column panels
+// (one slice per panel), and kRowBatch rows per thread for the sparse step
+// (whose untouched rows only decay).
 constexpr int kStateCols = 32;
 constexpr int kStateThreads = 256;
 constexpr int kMaxRowCtas = 1024;
@@ -81,6 +82,7 @@ struct Layout {
     // LM-head step (the gradient formed here on the tensor cores)
     size_t lm_colpart;  // float[ceil(V/128) * D]  sums of g^2 over each 128-row block
     size_t lm_rowpart;  // float[ceil(D/256) * V]  sums of g^2 over each 256-column block
+                        // (a dense step in column panels: over each panel)
     size_t total;
 };
 

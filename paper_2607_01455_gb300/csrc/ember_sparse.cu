@@ -33,7 +33,8 @@
 //   state     the dense step's column/normaliser pass, whose launch also runs
 //             the row pass: r for all V rows, the sums of new r per CTA, and
 //             the touched-row map cleared for the next step.
-//   apply     k_sp_apply: the update of the touched rows only.
+//   apply     k_sp_apply: the update of the touched rows only (once per
+//             column panel for tables wider than a CTA holds).
 //
 // Every kernel after the first is launched with programmatic dependent
 // launch and waits (griddepcontrol.wait) before it reads earlier results.
