@@ -229,6 +229,29 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     }
 }
 
+// beta2 r + (1 - beta2) m in fp32, each coefficient carried as a float pair
+// hi + lo (hi the coefficient rounded to fp32, lo the rest): within about an
+// ulp of the fp64 value, and the fixed point stays at r = m, which rounding
+// beta2 and 1 - beta2 to single floats would shift by about 1e-5 of r at
+// beta2 = 0.999.  With m = 0 (a row outside a sparse batch) it is the
+// correctly rounded product beta2 r in all but near-tie cases.
+struct EmaPair {
+    float bh, bl, ah, al;
+};
+__device__ __forceinline__ EmaPair make_ema_pair(double beta2, double one_minus_beta2)
+{
+    EmaPair e;
+    e.bh = (float)beta2;
+    e.bl = (float)(beta2 - (double)e.bh);
+    e.ah = (float)one_minus_beta2;
+    e.al = (float)(one_minus_beta2 - (double)e.ah);
+    return e;
+}
+__device__ __forceinline__ float ema_pair(const EmaPair &e, float r, float m)
+{
+    return fmaf(e.bh, r, fmaf(e.bl, r, fmaf(e.ah, m, e.al * m)));
+}
+
 // Pass 2: column EMA and the normaliser.  The first nstate CTAs each own
 // columns [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in
 // order.  For the sparse step the remaining CTAs also do the row pass: r for
@@ -304,19 +327,27 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
     } else {
         const int rb = (int)blockIdx.x - nstate;
         const int64_t stride = (int64_t)rowp.nrow_ctas * kStateThreads;
+        // This pass touches every row of the table, and GB300 runs fp64 at a
+        // small fraction of its fp32 rate: the row EMA runs in fp32 with its
+        // coefficients carried as float pairs (ema_pair), each thread adds
+        // its rows' new r in fp32, and only the sums across threads run in
+        // fp64.
+        const EmaPair ema = make_ema_pair(beta2, one_minus_beta2);
+        const float inv_Df = (float)inv_D;
         double rsum = 0.0;
         if (rowp.slot == nullptr) {
             // every row: per-column-block sums, slice-major, in block order
+            float tsum = 0.f;
             for (int64_t i = (int64_t)rb * kStateThreads + threadIdx.x; i < V; i += stride) {
                 float tot = 0.f;
 #pragma unroll 8
                 for (int k = 0; k < rowp.nslices; ++k)
                     tot += __ldcg(rowp.rowpart + (int64_t)k * V + i);
-                const double mean_row = (double)tot * inv_D;
-                const float rn = (float)(beta2 * (double)rowp.r[i] + one_minus_beta2 * mean_row);
+                const float rn = ema_pair(ema, rowp.r[i], tot * inv_Df);
                 rowp.r[i] = rn;
-                rsum += (double)rn;
+                tsum += rn;
             }
+            rsum = (double)tsum;
         } else {
             // sparse step: kRowBatch rows per thread at a time, their map
             // entries and r loaded together; rows outside the batch's ids
@@ -330,24 +361,26 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
                     sl[k] = (i < V) ? rowp.slot[i] : 0;
                     rr[k] = (i < V) ? rowp.r[i] : 0.f;
                 }
+                float tsum = 0.f;
 #pragma unroll
                 for (int k = 0; k < kRowBatch; ++k) {
                     const int64_t i = i0 + k * stride;
                     if (i >= V)
                         break;
-                    double mean_row = 0.0;
+                    float mean_row = 0.f;
                     if (sl[k]) {
                         const int64_t u = sl[k] - 1;
                         float tot = 0.f;
                         for (int q = 0; q < rowp.nslices; ++q)
                             tot += rowp.rowpart[u * rowp.nslices + q];
-                        mean_row = (double)tot * inv_D;
+                        mean_row = tot * inv_Df;
                         rowp.slot[i] = 0;
                     }
-                    const float rn = (float)(beta2 * (double)rr[k] + one_minus_beta2 * mean_row);
+                    const float rn = ema_pair(ema, rr[k], mean_row);
                     rowp.r[i] = rn;
-                    rsum += (double)rn;
+                    tsum += rn;
                 }
+                rsum += (double)tsum;
             }
         }
 #pragma unroll
