@@ -275,20 +275,25 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
     const int nstate = (int)gridDim.x - rowp.nrow_ctas;
-    __shared__ double part[kW][32];
+    __shared__ float part[kW][32];
+    __shared__ double part_last[kW][2];
     __shared__ bool am_last;
-    // means as products: fp64 division is a long instruction sequence, and
-    // the row pass of a sparse step runs it for every row of the table
+    // GB300 runs fp64 at a small fraction of its fp32 rate, and a single
+    // fp64 pipe op per row or column showed up in this kernel's time: the
+    // per-CTA work is fp32 (the EMAs with float-pair coefficients, sums of
+    // at most a few thousand values per CTA in fixed trees), and only the
+    // sums across CTAs and the normaliser run in fp64.
     const double inv_D = 1.0 / (double)D, inv_V = 1.0 / (double)V;
+    const EmaPair ema = make_ema_pair(beta2, one_minus_beta2);
     grid_dep_wait();  // column partials and row sums of the earlier passes
     grid_dep_launch();
 
     if ((int)blockIdx.x < nstate) {
         const int j = blockIdx.x * kStateCols + lane;
         // rows w, w + 8, w + 16, ...: 32 loads in flight, summed pairwise
-        // in fp32 within the batch and in fp64 across batches
+        // within the batch, then across batches and warps in order
         constexpr int kBatch = 32;
-        double acc = 0.0;
+        float acc = 0.f;
         if (j < D)
             for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
                 float v[kBatch];
@@ -302,39 +307,34 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
 #pragma unroll
                     for (int k = 0; k < h; ++k)
                         v[k] += v[k + h];
-                acc += (double)v[0];
+                acc += v[0];
             }
         part[w][lane] = acc;
         __syncthreads();
         if (w == 0) {
-            double tot = 0.0;
+            float tot = 0.f;
 #pragma unroll
             for (int q = 0; q < kW; ++q)
                 tot += part[q][lane];
-            double cn = 0.0;
+            float cn = 0.f;
             if (j < D) {
-                const double mean_col = tot * inv_V;
-                const float cnew = (float)(beta2 * (double)c[j] + one_minus_beta2 * mean_col);
+                const float cnew = ema_pair(ema, c[j], tot * (float)inv_V);
                 c[j] = cnew;
-                cn = (double)cnew;
+                cn = cnew;
             }
 #pragma unroll
             for (int o = 16; o >= 1; o >>= 1)
                 cn += __shfl_xor_sync(0xffffffffu, cn, o);
             if (lane == 0)
-                csum_part[blockIdx.x] = cn;
+                csum_part[blockIdx.x] = (double)cn;
         }
     } else {
         const int rb = (int)blockIdx.x - nstate;
         const int64_t stride = (int64_t)rowp.nrow_ctas * kStateThreads;
-        // This pass touches every row of the table, and GB300 runs fp64 at a
-        // small fraction of its fp32 rate: the row EMA runs in fp32 with its
-        // coefficients carried as float pairs (ema_pair), each thread adds
-        // its rows' new r in fp32, and only the sums across threads run in
-        // fp64.
-        const EmaPair ema = make_ema_pair(beta2, one_minus_beta2);
+        // Every row of the table: the row EMA (ema_pair), then the CTA's sum
+        // of the new r in fp32 (thread, warp butterfly, warps in order).
         const float inv_Df = (float)inv_D;
-        double rsum = 0.0;
+        float rsum = 0.f;
         if (rowp.slot == nullptr) {
             // every row: per-column-block sums, slice-major, in block order
             float tsum = 0.f;
@@ -347,7 +347,7 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
                 rowp.r[i] = rn;
                 tsum += rn;
             }
-            rsum = (double)tsum;
+            rsum = tsum;
         } else {
             // sparse step: kRowBatch rows per thread at a time, their map
             // entries and r loaded together; rows outside the batch's ids
@@ -380,7 +380,7 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
                     rowp.r[i] = rn;
                     tsum += rn;
                 }
-                rsum += (double)tsum;
+                rsum += tsum;
             }
         }
 #pragma unroll
@@ -390,10 +390,10 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
             part[w][0] = rsum;
         __syncthreads();
         if (threadIdx.x == 0) {
-            double t = 0.0;
+            float t = 0.f;
             for (int q = 0; q < kW; ++q)
                 t += part[q][0];
-            rsum_part[rb] = t;
+            rsum_part[rb] = (double)t;
         }
     }
     if (threadIdx.x == 0) {
@@ -419,16 +419,16 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
         rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
     }
     if (lane == 0) {
-        part[w][0] = csum;
-        part[w][1] = rsum;
+        part_last[w][0] = csum;
+        part_last[w][1] = rsum;
     }
     __syncthreads();
     if (threadIdx.x == 0) {
         csum = 0.0;
         rsum = 0.0;
         for (int q = 0; q < kW; ++q) {
-            csum += part[q][0];
-            rsum += part[q][1];
+            csum += part_last[q][0];
+            rsum += part_last[q][1];
         }
         const double rbar = rsum * inv_bc * inv_V;
         const double cbar = csum * inv_bc * inv_D;
