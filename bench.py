@@ -55,17 +55,6 @@ def step_bytes(wl):
     return (8 + 2 * w) * V * D + 8 * (V + D)
 
 
-def column_panels(D):
-    """Column panels the library splits a D-wide table into: a CTA holds
-    8192 columns of a row with 16-byte accesses (D % 4 == 0), 2048 without;
-    wider tables run in equal panels, one reduce and one apply launch each."""
-    vec = 4 if D % 4 == 0 else 1
-    maxw = 2048 * vec
-    n = -(-D // maxw)
-    pw = -(-(-(-D // n)) // vec) * vec
-    return -(-D // pw)
-
-
 def kernel_bytes(wl):
     """Algorithmic bytes per launch of each kernel of the dense step."""
     V, D, w = wl.V, wl.D, wbytes(wl)
@@ -181,7 +170,7 @@ def run_row_only(wl, dev, steps, warmup, flush, W, G):
         raise SystemExit("device status after the row-only steps")
     ms = sum(a.elapsed_time(b) for a, b in ev) / steps
     B = (4 + 2 * wbytes(wl)) * wl.V * wl.D + 8 * (wl.V + wl.D)
-    npan = column_panels(wl.D)
+    npan = emb.column_panels(wl.D % 4 == 0)
     # a table in column panels has no one-pass kernel: reduce, state and
     # apply passes per step, G read twice
     launches = 2 if npan == 1 else 2 * npan + 1
@@ -521,7 +510,8 @@ def run_ours(args, world, rank, local):
     G = synth.dense_grad(wl, rank, 1, dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
     emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
-    npan = column_panels(wl.D)
+    # column panels of this table (one reduce and one apply launch each)
+    npan = emb.column_panels(wl.D % 4 == 0)
 
     def one_step(t, ev):
         emb.trace(ev)

@@ -105,6 +105,15 @@ ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp,
 /* Free the host handle (never device memory).  NULL is ignored. */
 void ember_destroy(ember_handle *h);
 
+/* Column panels the dense, LM-head and sparse steps of this handle run in
+ * (see ember_create): 1 when a CTA holds a whole row, more for wider
+ * tables; each panel costs one reduce and one apply launch (one apply
+ * launch for the sparse and LM-head steps).  vector_path = 1 for pointers
+ * that take the 16-byte path (D % 4 == 0, W, G and rows 16-byte aligned,
+ * 8-byte for bf16 W), 0 for the scalar path.  Host only.  Returns 0 for a
+ * NULL handle. */
+int ember_column_panels(const ember_handle *h, int vector_path);
+
 /* Number of fp32 values of optimizer state: exactly V + D (Algorithm 1
  * keeps r in R^V and c in R^D).  The caller's state buffer holds r in
  * [0, V) followed by c in [V, V + D).  A new table starts from all zeros

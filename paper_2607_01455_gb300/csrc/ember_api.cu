@@ -114,6 +114,14 @@ ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp, ember_w
 
 void ember_destroy(ember_handle *h) { free(h); }
 
+int ember_column_panels(const ember_handle *h, int vector_path)
+{
+    ColMap m;
+    if (!h || !choose_colmap(h->D, vector_path != 0, &m))
+        return 0;
+    return m.npanels;
+}
+
 size_t ember_state_numel(const ember_handle *h)
 {
     return h ? (size_t)(h->V + h->D) : 0;

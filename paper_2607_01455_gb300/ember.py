@@ -40,6 +40,7 @@ EXPORTS = (
     "ember_step_dense_noalloc", "ember_step_dense_from_host",
     "ember_lmhead_grad", "ember_step_lmhead",
     "ember_shard_rows", "ember_shard_exchange_bytes", "ember_shard_reduce", "ember_shard_update",
+    "ember_column_panels",
 )
 
 
@@ -92,6 +93,7 @@ def lib():
             "ember_shard_exchange_bytes": (sz, [vp, ip]),
             "ember_shard_reduce": (st, [vp, ip, ip, vp, vp, vp, vp]),
             "ember_shard_update": (st, [vp, ip, ip, vp, vp, vp, vp, flt, i64, vp]),
+            "ember_column_panels": (ip, [vp, ip]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -129,6 +131,12 @@ def ember_status_string(status):
 
 def ember_abi_version():
     return lib().ember_abi_version()
+
+
+def ember_column_panels(h, vector_path=True):
+    """Column panels a step of this handle runs in (1 unless D is wider than
+    one CTA's row)."""
+    return lib().ember_column_panels(h, int(bool(vector_path)))
 
 
 def ember_hparams_default():
@@ -316,6 +324,9 @@ class Ember:
         ember_sparse_unique(self.handle, ids, idtype, n, uniq, counts, nu, stream)
         U = int(nu.item())
         return uniq[:U], counts[:U]
+
+    def column_panels(self, vector_path=True):
+        return ember_column_panels(self.handle, vector_path)
 
     def trace(self, events):
         ember_set_trace_events(self.handle, events)

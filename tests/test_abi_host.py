@@ -182,3 +182,20 @@ def test_step_and_bind_reject_on_host():
     finally:
         E.ember_destroy(h)
     E.ember_destroy(0)  # NULL is ignored
+
+
+@pytest.mark.parametrize("D", [1, 7, 2047, 2048, 2049, 3001, 4096, 8192, 8196, 10001, 12288, 16384,
+                               24576, 65533, 65536])
+def test_column_panels_follow_the_cta_row_width(D):
+    """A CTA holds 8192 columns of a row on the 16-byte path (D % 4 == 0),
+    2048 on the scalar one; a wider table runs in the fewest panels that
+    fit, ceil(D / width)."""
+    h = E.ember_create(3, D)
+    try:
+        vec = E.ember_column_panels(h, True)
+        sca = E.ember_column_panels(h, False)
+        assert sca == -(-D // 2048)
+        assert vec == (-(-D // 8192) if D % 4 == 0 else sca)
+    finally:
+        E.ember_destroy(h)
+    assert E.lib().ember_column_panels(None, 1) == 0
