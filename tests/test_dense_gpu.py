@@ -9,10 +9,9 @@ import numpy as np
 import pytest
 import torch
 
-import oracle
 from paper_2607_01455_gb300 import synth
 from paper_2607_01455_gb300.ember import Ember, EmberError
-from parity import Opt, check_state, check_weights, gated_dense_step, w_to_host
+from parity import Opt, gated_dense_step
 
 pytestmark = pytest.mark.gpu
 
