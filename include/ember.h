@@ -19,9 +19,12 @@
  *
  * Conventions shared by every entry point:
  *   - Device pointers are CUDA device (or managed) addresses on the current
- *     device; every array is row-major and contiguous.  The library never
- *     allocates or frees device memory: W, G, ids, rows, the state and the
- *     workspace belong to the caller.
+ *     device; every array is row-major and contiguous.  The library allocates
+ *     and frees no device memory at run time: W, G, ids, rows, the state and
+ *     the workspace belong to the caller.  The one exception is a static
+ *     10 MiB scratch array in the library's device code, present on every
+ *     GPU that loads the library until the process exits, which only
+ *     ember_step_dense_noalloc uses.
  *   - "stream" is a cudaStream_t passed as void* (NULL = the legacy default
  *     stream).  Steps are asynchronous on that stream.  Errors the host can
  *     see are returned at once and nothing is launched; errors only the GPU
@@ -32,8 +35,13 @@
  *     the workspace).
  *   - Results are deterministic: the same inputs give bit-identical W and
  *     state on every run.  No floating-point atomics are used; every sum is
- *     taken in a fixed order (the deterministic, atomic-free reduction that
- *     Section 2.3 asks for).
+ *     taken in a fixed order or, across CTAs, exactly in 64-bit fixed point
+ *     (the deterministic, atomic-free reduction that Section 2.3 asks for).
+ *   - Waits inside kernels are bounded (the mbarrier waits of the LM-head
+ *     kernel): a wait that runs past the handle's limit (2 s by default,
+ *     ember_set_wait_limit_ns) sets EMBER_ERR_TIMEOUT in the sticky device
+ *     flag and the kernel returns early, after the copies and matrix
+ *     operations it has issued complete; the step is then incomplete.
  */
 #ifndef EMBER_H
 #define EMBER_H
@@ -45,7 +53,7 @@
 extern "C" {
 #endif
 
-#define EMBER_ABI_VERSION 1
+#define EMBER_ABI_VERSION 2
 
 typedef enum {
     EMBER_OK = 0,
@@ -146,7 +154,14 @@ ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes
  *   lr:    step size alpha, applied in fp32 (any finite value).
  * W and G must be 4-byte (bf16 W: 2-byte) aligned; with D % 4 == 0 and
  * 16-byte aligned W, G and state the vectorised kernels run, otherwise a
- * scalar path gives the same results more slowly. */
+ * scalar path gives the same results more slowly.
+ *   A small table (V * D <= 65536 on the vector path, whose rows a CTA
+ * covers in a few passes) runs as one launch of a thread-block cluster of
+ * up to 8 CTAs that keeps G and W in shared memory and reads G from HBM
+ * once; every other table runs as three launches (reduce, column
+ * statistics and normaliser, update), chained with programmatic dependent
+ * launch.  Both forms run the same arithmetic on the same CTA row
+ * ranges and give the same bits.  Graph capture works for both. */
 ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *state,
                               float lr, int64_t t, void *stream);
 
@@ -175,11 +190,15 @@ ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G
  * a table processed in column panels (see ember_create) returns
  * EMBER_ERR_WORKSPACE.
  *   The first call on each device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call
- * before any stream capture.  All calls on a device share the one array and
- * each starts by zeroing its scalars, so calls that overlap on the GPU (two
- * streams, two handles, two threads) race and must be serialised by the
- * caller. */
+ * (cudaGetSymbolAddress) with that device current and caches it with the
+ * device's current CUDA context; it is looked up again if the context
+ * changes (after a cudaDeviceReset, for instance).  Make the first call on
+ * a device before any stream capture.  All calls on a device share the one
+ * array and each starts by zeroing its scalars, so calls that overlap on
+ * the GPU (two streams, two handles, two threads) race and must be
+ * serialised by the caller.  A timeout of a bounded wait is reported by
+ * the sticky flag in the array, which the next call clears: this entry
+ * point has no workspace for ember_get_device_status to read. */
 ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const float *G, float *state,
                                       float lr, int64_t t, void *stream);
 
@@ -217,48 +236,58 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
                                int64_t T, float *G, float *state, float lr, int64_t t, void *stream);
 
 /* Row-sharded dense step (Section 2.3: the statistics are sums of g^2, so
- * a table whose rows are spread over ranks needs only the per-rank partial
- * sums exchanged before the update).  A step is two calls per shard with
- * one exchange between them:
+ * a table whose rows are spread over ranks needs only small per-rank sums
+ * exchanged before the update: one value per column and one for the sum of
+ * r).  A step is three calls per shard with two all-reduces between them:
  *
- *   ember_shard_reduce  (every shard)  the reduction pass over the shard's
- *       rows: updates r for those rows and writes the shard's exchange block
- *       (its per-CTA column sums of g^2 and sums of new r);
- *   the caller all-gathers the blocks in shard order (NCCL all_gather of
- *       ember_shard_exchange_bytes per shard, or any copy);
- *   ember_shard_update  (every shard)  the column EMA and normaliser from all
- *       blocks (every shard forms the same c and s), then the update of the
+ *   ember_shard_reduce (every shard)  the reduction pass over the shard's
+ *       rows: updates r for those rows, keeps the shard's per-CTA partial
+ *       sums in its workspace, and writes `scales`: for each column (and, at
+ *       index D, for the sums of r) the largest fp32 exponent among the
+ *       shard's partials, one byte each;
+ *   the caller all-reduces `scales` with MAX (uint8, D + 1 bytes:
+ *       ember_shard_scale_bytes);
+ *   ember_shard_pack (every shard)  writes `sums`: each column's (and the r
+ *       sums') partials added in 64-bit fixed point at the all-reduced
+ *       exponent, one uint64 each;
+ *   the caller all-reduces `sums` with SUM (uint64/int64, 8 (D + 1) bytes:
+ *       ember_shard_exchange_bytes, 64 KiB at D = 8192);
+ *   ember_shard_update (every shard)  the column EMA and normaliser from the
+ *       totals (every shard forms the same c and s), then the update of the
  *       shard's rows of W.
  *
- * Shards are cut at the boundaries of the whole-table step's fixed CTA row
- * ranges, and every per-CTA partial is formed by the same kernel over the
- * same rows, so W, r and c come out bit-identical to ember_step_dense for
- * any number of shards (the paper's "bitwise identical" requirement of
- * Section 2.3).  The exchange holds one partial row per CTA (at most 304 x
- * D floats in all) rather than one reduced row, which is what keeps the
- * sum order independent of the shard count.
+ * Integer sums do not depend on how the partials are grouped, and the
+ * whole-table steps form the same fixed-point totals from the same per-CTA
+ * partials (shards are cut at the whole-table step's CTA row ranges), so W,
+ * r and c come out bit-identical to ember_step_dense for any number of
+ * shards (the paper's "bitwise identical" requirement of Section 2.3).
  *
  *   shard, nshards: 0 <= shard < nshards <= 4096.  Shards past the table's
- *       last CTA hold no rows (their calls still take part: the update
- *       maintains c).
+ *       last CTA hold no rows (their calls still take part: their scales
+ *       and sums are zero, and the update maintains c).
  *   G_shard, W_shard: the shard's rows (ember_shard_rows), row-major,
  *       device memory; with D % 4 == 0 they must be 16-byte aligned (8-byte
  *       for bf16 W) so that every shard takes the whole-table step's
  *       vector path (EMBER_ERR_ALIGNMENT otherwise).
  *   state: a full V + D buffer per shard; only the shard's rows of r and all
  *       of c are read and written.
- *   block: ember_shard_exchange_bytes(h, nshards) bytes, device, 256-byte
- *       aligned; blocks: nshards of them back to back, in shard order.
- * Variant ROW is not offered (EMBER_ERR_UNSUPPORTED): its one-pass kernel
- * needs no exchange for W and is run per shard with ember_step_dense.  Nor
- * are tables processed in column panels (see ember_create;
- * EMBER_ERR_UNSUPPORTED). */
+ *   scales: device, D + 1 bytes.  sums: device, D + 1 uint64, 8-byte
+ *       aligned.  Both caller-owned.
+ * Between a shard's reduce and its update the handle's workspace holds the
+ * shard's partials: run no other step of that handle in between.  Variant
+ * ROW is not offered (EMBER_ERR_UNSUPPORTED): its one-pass kernel needs no
+ * exchange for W and is run per shard with ember_step_dense.  Nor are tables
+ * processed in column panels (see ember_create; EMBER_ERR_UNSUPPORTED). */
 int64_t ember_shard_rows(const ember_handle *h, int shard, int nshards, int64_t *row0);
-size_t ember_shard_exchange_bytes(const ember_handle *h, int nshards);
+size_t ember_shard_scale_bytes(const ember_handle *h);
+size_t ember_shard_exchange_bytes(const ember_handle *h);
 ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const float *G_shard, float *state,
-                                void *block, void *stream);
+                                unsigned char *scales, void *stream);
+ember_status ember_shard_pack(ember_handle *h, int shard, int nshards, const unsigned char *scales,
+                              unsigned long long *sums, void *stream);
 ember_status ember_shard_update(ember_handle *h, int shard, int nshards, void *W_shard, const float *G_shard,
-                                float *state, const void *blocks, float lr, int64_t t, void *stream);
+                                float *state, const unsigned char *scales, const unsigned long long *sums,
+                                float lr, int64_t t, void *stream);
 
 /* One sparse Ember step (Section 2.2) at step number t >= 1.
  *   ids:   N token ids of type idtype (duplicates allowed, any order).
@@ -300,6 +329,14 @@ ember_status ember_get_device_status(ember_handle *h, void *stream);
  * events = NULL or n = 0 to stop tracing.  The events are not recorded
  * when n is too small for a step; nothing else changes. */
 ember_status ember_set_trace_events(ember_handle *h, void *const *events, int n);
+
+/* Limit, in nanoseconds of wall time, of the bounded waits inside this
+ * handle's kernels (the main-loop mbarrier waits of the LM-head kernel; its
+ * teardown waits keep 2 s so that copies already issued always complete);
+ * 0 restores the default of 2 s.  A short limit makes a wait give up on
+ * purpose: the kernel sets EMBER_ERR_TIMEOUT and returns early, which is how
+ * the failure path is tested.  Host only. */
+ember_status ember_set_wait_limit_ns(ember_handle *h, uint64_t ns);
 
 /* Static description of a status code. */
 const char *ember_status_string(ember_status s);

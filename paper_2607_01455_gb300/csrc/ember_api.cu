@@ -24,7 +24,7 @@ Layout make_layout(int64_t V, int64_t D, int64_t max_sparse_N)
     };
     const size_t nstate = (size_t)((D + kStateCols - 1) / kStateCols);
     L.scalars = take(sizeof(DevScalars));
-    L.rsum_part = take(sizeof(double) * kRsumParts);
+    L.rsum_part = take(sizeof(float) * kRsumParts);
     L.csum_part = take(sizeof(double) * nstate);
     L.colpart = take(sizeof(float) * (size_t)kPartRows * (size_t)D);
     if (max_sparse_N > 0) {
@@ -108,6 +108,7 @@ ember_status ember_create(int64_t V, int64_t D, const ember_hparams *hp, ember_w
     e->D = D;
     e->hp = h;
     e->wdtype = wdtype;
+    e->wait_ns = kDefaultWaitNs;
     *out = e;
     return EMBER_OK;
 }
@@ -195,6 +196,7 @@ ember_status ember_step_dense(ember_handle *h, void *W, const float *G, float *s
     a.lay = make_layout(h->V, h->D, h->ws_max_N);
     a.stream = (cudaStream_t)stream;
     a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    a.wait_ns = h->wait_ns;
     const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && is_aligned(G, 16);
     if (!choose_colmap(h->D, vec4, &a.map))
         return EMBER_ERR_UNSUPPORTED;
@@ -244,6 +246,7 @@ ember_status ember_step_dense_from_host(ember_handle *h, void *W, const float *G
     a.lay = make_layout(h->V, h->D, h->ws_max_N);
     a.stream = (cudaStream_t)stream;
     a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    a.wait_ns = h->wait_ns;
     const bool vec4 = (h->D % 4 == 0) && is_aligned(W, 4 * wsz) && is_aligned(G_dev, 16) &&
                       is_aligned(G_stage, 16);
     if (!choose_colmap(h->D, vec4, &a.map))
@@ -274,7 +277,7 @@ ember_status ember_lmhead_grad(ember_handle *h, const void *dlogits, const void 
     if (st != EMBER_OK)
         return st;
     const Layout L = make_layout(h->V, h->D, h->ws_max_N);
-    LmArgs lm{h->V, h->D, T, dlogits, hidden, G};
+    LmArgs lm{h->V, h->D, T, dlogits, hidden, G, h->wait_ns};
     DevScalars *sc = reinterpret_cast<DevScalars *>(h->ws + L.scalars);
     const cudaError_t e = launch_lmhead_grad(lm, reinterpret_cast<float *>(h->ws + L.lm_colpart),
                                              reinterpret_cast<float *>(h->ws + L.lm_rowpart), &sc->flags,
@@ -296,7 +299,7 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
     if (!is_aligned(W, wsz) || !is_aligned(state, 4))
         return EMBER_ERR_ALIGNMENT;
 
-    LmArgs lm{h->V, h->D, T, dlogits, hidden, G};
+    LmArgs lm{h->V, h->D, T, dlogits, hidden, G, h->wait_ns};
     DenseArgs a{};
     a.V = h->V;
     a.D = h->D;
@@ -315,6 +318,7 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
     a.lay = make_layout(h->V, h->D, h->ws_max_N);
     a.stream = (cudaStream_t)stream;
     a.trace = (h->n_trace >= 4) ? h->trace : nullptr;
+    a.wait_ns = h->wait_ns;
     a.lm = &lm;
     const bool vec4 = is_aligned(W, 4 * wsz);  // D % 8 == 0 and G 16-byte aligned already
     if (!choose_colmap(h->D, vec4, &a.map))
@@ -324,13 +328,11 @@ ember_status ember_step_lmhead(ember_handle *h, void *W, const void *dlogits, co
 
 // ---- row-sharded dense step ----
 
-static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
-
 static bool shard_plan(const ember_handle *h, int shard, int nshards, ShardArgs *p)
 {
     if (!h || nshards < 1 || nshards > kMaxShards || shard < 0 || shard >= nshards)
         return false;
-    const int nparts = dense_parts(h->V);
+    const int nparts = dense_parts(h->V, h->D);
     const int cap = (nparts + nshards - 1) / nshards;
     int b0 = shard * cap, b1 = (shard + 1) * cap;
     if (b0 > nparts)
@@ -339,11 +341,7 @@ static bool shard_plan(const ember_handle *h, int shard, int nshards, ShardArgs 
         b1 = nparts;
     p->cta_begin = b0;
     p->cta_end = b1;
-    p->cap = cap;
-    p->nshards = nshards;
     p->row_base = (int64_t)b0 * h->V / nparts;
-    p->block_rsum = align256(sizeof(float) * (size_t)cap * (size_t)h->D);
-    p->block_bytes = p->block_rsum + align256(sizeof(double) * (size_t)cap);
     return true;
 }
 
@@ -352,38 +350,36 @@ int64_t ember_shard_rows(const ember_handle *h, int shard, int nshards, int64_t 
     ShardArgs p{};
     if (!shard_plan(h, shard, nshards, &p))
         return -1;
-    const int nparts = dense_parts(h->V);
+    const int nparts = dense_parts(h->V, h->D);
     const int64_t r1 = (int64_t)p.cta_end * h->V / nparts;
     if (row0)
         *row0 = p.row_base;
     return r1 - p.row_base;
 }
 
-size_t ember_shard_exchange_bytes(const ember_handle *h, int nshards)
+size_t ember_shard_scale_bytes(const ember_handle *h) { return h ? (size_t)(h->D + 1) : 0; }
+
+size_t ember_shard_exchange_bytes(const ember_handle *h)
 {
-    ShardArgs p{};
-    if (!shard_plan(h, 0, nshards, &p))
-        return 0;
-    return p.block_bytes;
+    return h ? sizeof(unsigned long long) * (size_t)(h->D + 1) : 0;
 }
 
+// Checks shared by the three phases; fills the plan and the common step
+// arguments.  G_shard / W_shard are checked only when given (non-null).
 static ember_status shard_common(ember_handle *h, int shard, int nshards, const void *W_shard, const float *G_shard,
-                                 const float *state, const void *block, ShardArgs *p, DenseArgs *a)
+                                 const float *state, ShardArgs *p, DenseArgs *a)
 {
-    if (!h || !state || !block)
+    if (!h || !state)
         return EMBER_ERR_INVALID_ARG;
     if (!shard_plan(h, shard, nshards, p))
-        return EMBER_ERR_INVALID_ARG;
-    const bool has_rows = p->cta_end > p->cta_begin;
-    if (has_rows && !G_shard)
         return EMBER_ERR_INVALID_ARG;
     if (h->hp.variant == EMBER_VARIANT_ROW)
         return EMBER_ERR_UNSUPPORTED;  // the row-only step has its own one-pass kernel
     // every shard must take the same vector path as the whole-table step
     const size_t wsz = h->wdtype == EMBER_BF16 ? 2 : 4;
     const bool vec4 = h->D % 4 == 0;
-    if (!is_aligned(state, 4) || !is_aligned(block, 256) ||
-        (has_rows && (!is_aligned(G_shard, vec4 ? 16 : 4) || (W_shard && !is_aligned(W_shard, vec4 ? 4 * wsz : wsz)))))
+    if (!is_aligned(state, 4) || (G_shard && !is_aligned(G_shard, vec4 ? 16 : 4)) ||
+        (W_shard && !is_aligned(W_shard, vec4 ? 4 * wsz : wsz)))
         return EMBER_ERR_ALIGNMENT;
     if (!h->ws)
         return EMBER_ERR_WORKSPACE;
@@ -400,6 +396,7 @@ static ember_status shard_common(ember_handle *h, int shard, int nshards, const 
     a->ws = h->ws;
     a->lay = make_layout(h->V, h->D, h->ws_max_N);
     a->trace = nullptr;
+    a->wait_ns = h->wait_ns;
     if (!choose_colmap(h->D, vec4, &a->map))
         return EMBER_ERR_UNSUPPORTED;
     if (a->map.npanels != 1)
@@ -408,15 +405,43 @@ static ember_status shard_common(ember_handle *h, int shard, int nshards, const 
 }
 
 ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const float *G_shard, float *state,
-                                void *block, void *stream)
+                                unsigned char *scales, void *stream)
 {
     ShardArgs p{};
     DenseArgs a{};
-    const ember_status st = shard_common(h, shard, nshards, nullptr, G_shard, state, block, &p, &a);
+    if (!scales)
+        return EMBER_ERR_INVALID_ARG;
+    const ember_status st = shard_common(h, shard, nshards, nullptr, G_shard, state, &p, &a);
     if (st != EMBER_OK)
         return st;
+    if (p.cta_end > p.cta_begin && !G_shard)
+        return EMBER_ERR_INVALID_ARG;
     p.phase = 1;
-    p.block = block;
+    p.scales = scales;
+    a.shard = &p;
+    a.inv_bc = 1.0;
+    a.stream = (cudaStream_t)stream;
+    return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
+}
+
+ember_status ember_shard_pack(ember_handle *h, int shard, int nshards, const unsigned char *scales,
+                              unsigned long long *sums, void *stream)
+{
+    ShardArgs p{};
+    DenseArgs a{};
+    if (!h || !scales || !sums)
+        return EMBER_ERR_INVALID_ARG;
+    if (!is_aligned(sums, 8))
+        return EMBER_ERR_ALIGNMENT;
+    // the state is not touched by this phase; any aligned non-null pointer
+    // passes the shared checks
+    const ember_status st = shard_common(h, shard, nshards, nullptr, nullptr, reinterpret_cast<float *>(sums), &p,
+                                         &a);
+    if (st != EMBER_OK)
+        return st;
+    p.phase = 2;
+    p.scales = const_cast<unsigned char *>(scales);
+    p.sums = sums;
     a.shard = &p;
     a.inv_bc = 1.0;
     a.stream = (cudaStream_t)stream;
@@ -424,20 +449,26 @@ ember_status ember_shard_reduce(ember_handle *h, int shard, int nshards, const f
 }
 
 ember_status ember_shard_update(ember_handle *h, int shard, int nshards, void *W_shard, const float *G_shard,
-                                float *state, const void *blocks, float lr, int64_t t, void *stream)
+                                float *state, const unsigned char *scales, const unsigned long long *sums, float lr,
+                                int64_t t, void *stream)
 {
     if (t < 1 || !isfinite(lr))
         return EMBER_ERR_INVALID_ARG;
+    if (!scales || !sums)
+        return EMBER_ERR_INVALID_ARG;
+    if (!is_aligned(sums, 8))
+        return EMBER_ERR_ALIGNMENT;
     ShardArgs p{};
     DenseArgs a{};
     a.W = W_shard;
-    const ember_status st = shard_common(h, shard, nshards, W_shard, G_shard, state, blocks, &p, &a);
+    const ember_status st = shard_common(h, shard, nshards, W_shard, G_shard, state, &p, &a);
     if (st != EMBER_OK)
         return st;
-    if (p.cta_end > p.cta_begin && !W_shard)
+    if (p.cta_end > p.cta_begin && (!W_shard || !G_shard))
         return EMBER_ERR_INVALID_ARG;
-    p.phase = 2;
-    p.blocks = blocks;
+    p.phase = 3;
+    p.scales = const_cast<unsigned char *>(scales);
+    p.sums = const_cast<unsigned long long *>(sums);
     a.shard = &p;
     a.inv_bc = h->hp.bias_correction ? 1.0 / (1.0 - pow(h->hp.beta2, (double)t)) : 1.0;
     a.lr_signed = h->hp.maximize ? lr : -lr;
@@ -536,10 +567,24 @@ ember_status ember_get_device_status(ember_handle *h, void *stream)
     if (flags && (cudaMemsetAsync(&sc->flags, 0, sizeof(unsigned), s) != cudaSuccess ||
                   cudaStreamSynchronize(s) != cudaSuccess))
         return EMBER_ERR_CUDA;
+    // a wait that gave up leaves the grid-barrier words of the one-launch
+    // steps set (abort, partial arrivals): clear them so the next step runs
+    if ((flags & kFlagTimeout) &&
+        (cudaMemsetAsync(&sc->bar_count, 0, 4 * sizeof(unsigned), s) != cudaSuccess ||
+         cudaStreamSynchronize(s) != cudaSuccess))
+        return EMBER_ERR_CUDA;
     if (flags & kFlagTimeout)
         return EMBER_ERR_TIMEOUT;
     if (flags & kFlagIdRange)
         return EMBER_ERR_ID_OUT_OF_RANGE;
+    return EMBER_OK;
+}
+
+ember_status ember_set_wait_limit_ns(ember_handle *h, uint64_t ns)
+{
+    if (!h)
+        return EMBER_ERR_INVALID_ARG;
+    h->wait_ns = ns ? ns : kDefaultWaitNs;
     return EMBER_OK;
 }
 

@@ -3,39 +3,54 @@
 //
 // The step needs two passes over the fp32 gradient G: the update of any
 // element needs chat_j and s, which depend on every row of G (Section 2.3
-// builds both statistics from sums of g^2).  The passes are:
+// builds both statistics from sums of g^2).  The work is:
 //
-//   reduce  (k_reduce_dense)  one read of G.  Per row: sum_j g^2, the row EMA
+//   reduce  one read of G.  Per row: sum_j g^2 and the row EMA
 //           r_i <- beta2 r_i + (1-beta2) mean_j g^2 (Algorithm 1's row second
 //           moment), written once.  Per CTA: column sums of g^2 over its rows
 //           and the sum of its new r values, written to the workspace.
-//   state   (k_state_dense)   O(D * CTAs) work: column sums in a fixed order,
-//           the column EMA c_j <- beta2 c_j + (1-beta2) mean_i g^2, then the
-//           last CTA forms mean(rhat), mean(chat) and s = sqrt(mean rhat *
-//           mean chat) (the geometric-mean normaliser).
-//   apply   (k_apply_dense)   reads G and W, writes W:
+//   state   O(D * CTAs) work: per column the exact fixed-point total of the
+//           per-CTA partial sums (ember_device.cuh), the column EMA
+//           c_j <- beta2 c_j + (1-beta2) mean_i g^2; then mean(rhat),
+//           mean(chat) and s = sqrt(mean rhat * mean chat) (the
+//           geometric-mean normaliser).
+//   apply   reads G and W, writes W:
 //           W_ij <- W_ij - lr g_ij / (sqrt(rhat_i) sqrt(chat_j / s) + eps),
 //           the factored preconditioner applied as a row scale times a
 //           column scale, never stored (Section 2.3).
 //
+// By default the three parts run as ONE cooperative launch (k_dense_fused):
+// every CTA reduces its rows, a grid barrier, the CTAs share the column
+// groups, a second grid barrier, then every CTA forms s itself (the same
+// arithmetic in every CTA) and updates its rows.  The barriers replace two
+// kernel boundaries, which is what small and mid-size tables pay for most.
+// The three-kernel form (k_reduce_dense, k_state_dense, k_apply_dense) runs
+// the same device code on the same CTA grid and gives the same bits; it
+// serves the steps that need more than one launch anyway (column panels,
+// the LM-head step, row shards, a gradient in host memory), traced steps,
+// and devices where the cooperative grid does not fit.
+//
 // Bandwidth: 4VD bytes (reduce) + 4VD + 2 w VD bytes (apply), w = bytes per
-// weight.  The apply pass walks each CTA's rows in the reverse order of the
-// reduce pass, so the rows read last by the reduce pass -- still in L2 --
-// are the first ones it needs.
+// weight.  The apply walks each CTA's rows in the reverse order of the
+// reduce, so the rows read last by the reduce -- still in L2 -- are the first
+// ones it needs.
 //
 // Determinism: no floating-point atomics.  Every CTA owns a fixed row range
-// (a function of V only), every in-CTA sum has a fixed shape, and the
-// cross-CTA sums run in CTA order, so W and the state are bit-identical
-// from run to run, as Section 2.3 requires.
+// (a function of V and D only) and every in-CTA sum has a fixed shape; the
+// sums across CTAs are exact integer sums, so W and the state are
+// bit-identical from run to run and however the partials are grouped (the
+// row-sharded step relies on that), as Section 2.3 requires.
 //
 // The same launcher also runs:
 //   - the row-only variant in one pass (k_rowonly_dense), no apply pass;
 //   - the LM-head step: the tensor-core kernel of ember_lmhead.cu forms G and
 //     its per-tile sums of g^2, the state pass finishes them (row pass from
 //     per-column-block sums), then the apply pass;
-//   - the two phases of a row-sharded step: the reduce pass or the apply
-//     pass over one shard's CTAs of the whole-table grid (RowSpan), and the
-//     state pass on every shard's gathered partials.
+//   - the three phases of a row-sharded step: the reduce over one shard's
+//     CTAs of the whole-table grid (RowSpan) with the shard's largest
+//     exponents per column, the fixed-point pack at the all-reduced
+//     exponents, and the state pass on the all-reduced totals followed by
+//     the shard's apply;
 //   - tables wider than a CTA holds (more than 8192 columns, or 2048 without
 //     16-byte accesses): the reduce and apply passes once per column panel
 //     with the row stride D, the rows' sums of g^2 per panel added up by the
@@ -52,20 +67,36 @@ namespace {
 
 using namespace dev;
 
-// Pass 1: one read of G.  Template: VEC columns per access, CPT accesses per
-// thread per row, R rows per row group per iteration.
+// beta2 r + (1 - beta2) m in fp32 with the coefficients carried as float
+// pairs (StepConsts): within about an ulp of the fp64 value, and the fixed
+// point stays at r = m, which rounding beta2 and 1 - beta2 to single floats
+// would shift by about 1e-5 of r at beta2 = 0.999.  With m = 0 (a row outside
+// a sparse batch) it is the correctly rounded product beta2 r in all but
+// near-tie cases.
+__device__ __forceinline__ float ema_pair(const EmaPair &e, float r, float m)
+{
+    return fmaf(e.bh, r, fmaf(e.bl, r, fmaf(e.ah, m, e.al * m)));
+}
+
+// ---------------------------------------------------------------------------
+// Reduce: one read of G.  VEC columns per access, CPT accesses per thread per
+// row, R rows per row group per iteration.  The CTA's rows are those of CTA
+// span.cta_base + cta of a grid of span.nparts over the table; its column
+// partial goes to colpart_row, the sum of its new r to *rsum_out.
 // STAGE: G is read from host memory the GPU can address (over the
 // Grace-Blackwell chip-to-chip link) and every element is also written to
 // G_stage in HBM for the apply pass.
 // D is the number of columns this launch covers and ld the row stride of G
 // and colpart: a column panel of a wider table has D < ld, and then each
 // row's sum of g^2 over the panel goes to rowpart[i] instead of into r.
-template <int VEC, int CPT, int R, bool STAGE>
-__global__ void __launch_bounds__(kThreads, kCtasPerSm)
-k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
-               float *__restrict__ colpart, double *__restrict__ rsum_part,
-               int64_t V, int D, int ld, int tpr, double beta2, double one_minus_beta2,
-               float *__restrict__ G_stage, float *__restrict__ rowpart, RowSpan span)
+// ---------------------------------------------------------------------------
+template <int VEC, int CPT, int R, bool STAGE, bool KEEP = false>
+__device__ __forceinline__ void reduce_rows(const float *__restrict__ G, float *__restrict__ r,
+                                            float *__restrict__ colpart_row, float *__restrict__ rsum_out,
+                                            int64_t V, int D, int ld, int tpr, const StepConsts &kc,
+                                            float *__restrict__ G_stage, float *__restrict__ rowpart,
+                                            RowSpan span, int cta,
+                                            float *__restrict__ comb, typename Vec<VEC>::F *__restrict__ keep)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
@@ -77,16 +108,13 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     const int g = tid / tpr;                 // this thread's row group
     const int l = tid - g * tpr;             // position within the row
     const int wpg = tpr >> 5;                // warps per row group
-    const int64_t row0 = (int64_t)(span.cta_base + blockIdx.x) * V / span.nparts;
-    const int64_t row1 = (int64_t)(span.cta_base + blockIdx.x + 1) * V / span.nparts;
-
-    grid_dep_wait();    // the first kernel of a step: returns at once
-    grid_dep_launch();  // the state pass may start launching now; it waits for this grid
+    const int64_t row0 = (int64_t)(span.cta_base + cta) * V / span.nparts;
+    const int64_t row1 = (int64_t)(span.cta_base + cta + 1) * V / span.nparts;
 
     // per-warp row sums of up to kRowBuf rows, finalised together
     constexpr int kRowBuf = 128;
     __shared__ float red[kWarps][kRowBuf];
-    __shared__ double rsum_sh[kWarps];
+    __shared__ float rsum_sh[kWarps];
 
     float acc[CPT][VEC];
 #pragma unroll
@@ -94,13 +122,14 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
             acc[c][e] = 0.f;
-    double rsum = 0.0;
+    float rsum = 0.f;
 
-    const int rows_per_it = rg * R;               // rows of one iteration
+    const int rows_per_it = rg * R;                 // rows of one iteration
     const int its_per_buf = kRowBuf / rows_per_it;  // >= 1: rg * R <= 128
     int64_t buf_base = row0;
     int nbuf = 0;  // iterations held in the buffer
-    for (int64_t base = row0; base < row1; base += rows_per_it) {
+    int it = 0;    // iteration index (the slot of the kept G)
+    for (int64_t base = row0; base < row1; base += rows_per_it, ++it) {
         F v[R][CPT];
 #pragma unroll
         for (int k = 0; k < R; ++k) {
@@ -118,6 +147,8 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                     v[k][c] = in ? load_g<VEC>(G + (i - span.row_base) * ld + (int64_t)col * VEC)
                                  : zero_vec<VEC>();
                 }
+                if constexpr (KEEP)  // this thread's slot of the iteration, read back by the update
+                    keep[((it * R + k) * CPT + c) * kThreads + tid] = v[k][c];
             }
         }
         // squares and per-row partial sums
@@ -172,10 +203,9 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
                         rowpart[i] = sum;
                         continue;
                     }
-                    const double mean_row = (double)sum / (double)D;
-                    const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
+                    const float rn = ema_pair(kc.ema, r[i], sum * kc.inv_D);
                     r[i] = rn;
-                    rsum += (double)rn;
+                    rsum += rn;
                 }
             }
             __syncthreads();
@@ -185,7 +215,6 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
     }
 
     // column partial of this CTA: row groups combined in order 0 .. rg-1
-    float *out = colpart + (int64_t)blockIdx.x * ld;
     if (rg == 1) {
 #pragma unroll
         for (int c = 0; c < CPT; ++c) {
@@ -193,10 +222,10 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
             if (col < DV)
 #pragma unroll
                 for (int e = 0; e < VEC; ++e)
-                    out[col * VEC + e] = acc[c][e];
+                    colpart_row[col * VEC + e] = acc[c][e];
         }
     } else {
-        extern __shared__ float colsh[];  // D floats
+        float *colsh = comb;  // D floats of shared memory
         for (int q = 0; q < rg; ++q) {
             if (g == q) {
 #pragma unroll
@@ -211,10 +240,11 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
             __syncthreads();
         }
         for (int j = tid; j < D; j += kThreads)
-            out[j] = colsh[j];
+            colpart_row[j] = colsh[j];
     }
 
-    // sum of the new r values of this CTA: fixed butterfly per warp, warps in order
+    // sum of the new r values of this CTA (fp32): fixed butterfly per warp,
+    // warps in order
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
         rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
@@ -222,42 +252,311 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r,
         rsum_sh[warp] = rsum;
     __syncthreads();
     if (tid == 0 && rowpart == nullptr) {
-        double s = 0.0;
+        float s = 0.f;
         for (int q = 0; q < kWarps; ++q)
             s += rsum_sh[q];
-        rsum_part[blockIdx.x] = s;
+        *rsum_out = s;
     }
 }
 
-// beta2 r + (1 - beta2) m in fp32, each coefficient carried as a float pair
-// hi + lo (hi the coefficient rounded to fp32, lo the rest): within about an
-// ulp of the fp64 value, and the fixed point stays at r = m, which rounding
-// beta2 and 1 - beta2 to single floats would shift by about 1e-5 of r at
-// beta2 = 0.999.  With m = 0 (a row outside a sparse batch) it is the
-// correctly rounded product beta2 r in all but near-tie cases.
-struct EmaPair {
-    float bh, bl, ah, al;
-};
-__device__ __forceinline__ EmaPair make_ema_pair(double beta2, double one_minus_beta2)
+// ---------------------------------------------------------------------------
+// Apply: the update of the CTA's rows, walked from the last iteration block
+// to the first.  The column scales live in shared memory (D floats): cs[j] =
+// sqrt(chat_j / s) (FULL), sqrt(chat_j) (COL) or 1 (ROW).  D columns from row
+// stride ld, as in the reduce: W, G and c point at the first column of the
+// panel.  r and c are read through L2 (they may have been written earlier in
+// the same launch).
+// ---------------------------------------------------------------------------
+template <int VEC, int CPT, int R, bool BF16>
+__device__ __forceinline__ void apply_rows(void *__restrict__ W, const float *__restrict__ G,
+                                           const float *__restrict__ r, const float *__restrict__ c,
+                                           float inv_s_full, int64_t V, int D, int ld, int tpr, float inv_bc,
+                                           float eps, float lr_signed, int variant, RowSpan span, int cta)
 {
-    EmaPair e;
-    e.bh = (float)beta2;
-    e.bl = (float)(beta2 - (double)e.bh);
-    e.ah = (float)one_minus_beta2;
-    e.al = (float)(one_minus_beta2 - (double)e.ah);
-    return e;
-}
-__device__ __forceinline__ float ema_pair(const EmaPair &e, float r, float m)
-{
-    return fmaf(e.bh, r, fmaf(e.bl, r, fmaf(e.ah, m, e.al * m)));
+    using F = typename Vec<VEC>::F;
+    using WT = typename WRaw<BF16, VEC>::T;
+    extern __shared__ float cs[];  // D column scales
+    const int DV = D / VEC;
+    const int tid = threadIdx.x;
+    const int rg = kThreads / tpr;
+    const int g = tid / tpr;
+    const int l = tid - g * tpr;
+    const int64_t row0 = (int64_t)(span.cta_base + cta) * V / span.nparts;
+    const int64_t row1 = (int64_t)(span.cta_base + cta + 1) * V / span.nparts;
+    const int64_t step = (int64_t)rg * R;
+    const int64_t nblocks = (row1 - row0 + step - 1) / step;
+
+    const float inv_s = (variant == EMBER_VARIANT_FULL) ? inv_s_full : 1.f;
+    for (int j = tid; j < D; j += kThreads)
+        cs[j] = (variant == EMBER_VARIANT_ROW) ? 1.f : sqrtf(__ldcg(c + j) * inv_bc * inv_s);
+    __syncthreads();
+
+    for (int64_t b = nblocks - 1; b >= 0; --b) {
+        const int64_t base = row0 + b * step;
+        F gv[R][CPT];
+        WT wr[R][CPT];
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+#pragma unroll
+            for (int cc = 0; cc < CPT; ++cc) {
+                const int col = l + cc * tpr;
+                if (i < row1 && col < DV) {
+                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
+                    gv[k][cc] = load_g<VEC>(G + idx);
+                    wr[k][cc] = load_w<BF16, VEC>(W, idx);
+                }
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = base + (int64_t)g * R + k;
+            if (i >= row1)
+                continue;
+            const float rs = (variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(__ldcg(r + i) * inv_bc);
+#pragma unroll
+            for (int cc = 0; cc < CPT; ++cc) {
+                const int col = l + cc * tpr;
+                if (col >= DV)
+                    continue;
+                float w[VEC];
+                unpack_w(wr[k][cc], w);
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const float den = fmaf(rs, cs[col * VEC + e], eps);
+                    const float u = comp(gv[k][cc], e) / den;
+                    w[e] = fmaf(lr_signed, u, w[e]);
+                }
+                store_w<BF16, VEC>(W, (i - span.row_base) * ld + (int64_t)col * VEC, w);
+            }
+        }
+    }
 }
 
-// Pass 2: column EMA and the normaliser.  The first nstate CTAs each own
-// columns [32x, 32x + 32); warp w sums the partials of CTAs w, w+8, ... in
-// order.  For the sparse step the remaining CTAs also do the row pass: r for
-// every row (rows outside the batch see a zero gradient row, touched rows
-// take their sum of g^2 per column slice from `rowpart`) and the sum of the
-// new r per CTA.  The last CTA to finish forms mean(rhat), mean(chat) and s.
+// ---------------------------------------------------------------------------
+// Column pass of one group of kStateCols = 32 columns, by a whole CTA of
+// kStateThreads threads: lane l of every warp owns column j0 + l.
+// Source: the partial rows colpart[b * D + j], b < nparts (warp w reads rows
+// w, w + 8, ...; the column's total is their exact fixed-point sum at the
+// largest key among them), or, with `sums` set, the totals already formed
+// elsewhere (the all-reduce of a row-sharded step) at scales[j].
+// Writes c_j <- beta2 c_j + (1 - beta2) total_j / V and csum_part[group] =
+// the fp32 sum of the group's new c (a fixed butterfly).
+// ---------------------------------------------------------------------------
+struct ColSource {
+    const float *colpart;                 // [nparts][D]
+    int nparts;
+    const unsigned long long *sums;       // nullptr, or [D] totals
+    const unsigned char *scales;          // their scale exponents
+};
+
+constexpr int kStateWarps = kStateThreads / 32;
+// partial rows per warp held in registers by the column pass (304 rows of
+// the dense step fit; more, as the LM-head and sparse steps have, take two
+// passes through L2)
+constexpr int kRegParts = 38;
+static_assert(kRegParts * kStateWarps >= kGridCtas, "the dense step's partial rows fit the register path");
+
+__device__ __forceinline__ void column_group(const ColSource &src, int group, float *__restrict__ c,
+                                             float *__restrict__ csum_part, int D, const StepConsts &kc)
+{
+    __shared__ unsigned emax_sh[kStateWarps][32];
+    __shared__ unsigned long long ssum_sh[kStateWarps][32];
+    const int lane = threadIdx.x & 31;
+    const int w = threadIdx.x >> 5;
+    const int j = group * kStateCols + lane;
+    unsigned long long S = 0;
+    unsigned E = 0;
+    if (src.sums == nullptr && src.nparts <= kRegParts * kStateWarps) {
+        // up to kRegParts partial rows per warp: one trip to L2, the values
+        // kept in registers for both the largest key and the sum
+        float v[kRegParts];
+        unsigned e = 0;
+#pragma unroll
+        for (int k = 0; k < kRegParts; ++k) {
+            const int b = w + k * kStateWarps;
+            v[k] = (b < src.nparts && j < D) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+        }
+#pragma unroll
+        for (int k = 0; k < kRegParts; ++k)
+            e = max(e, fx_key(v[k]));
+        emax_sh[w][lane] = e;
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < kStateWarps; ++q)
+            E = max(E, emax_sh[q][lane]);
+        unsigned long long s = 0;
+#pragma unroll
+        for (int k = 0; k < kRegParts; ++k)
+            s += fx_of(v[k], E);
+        ssum_sh[w][lane] = s;
+        __syncthreads();
+        if (w == 0)
+#pragma unroll
+            for (int q = 0; q < kStateWarps; ++q)
+                S += ssum_sh[q][lane];
+    } else if (src.sums == nullptr) {
+        constexpr int kBatch = 16;
+        // pass 1: the largest key of the column (loads batched for latency)
+        unsigned e = 0;
+        if (j < D)
+            for (int b0 = w; b0 < src.nparts; b0 += kBatch * kStateWarps) {
+                float v[kBatch];
+#pragma unroll
+                for (int k = 0; k < kBatch; ++k) {
+                    const int b = b0 + k * kStateWarps;
+                    v[k] = (b < src.nparts) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+                }
+#pragma unroll
+                for (int k = 0; k < kBatch; ++k)
+                    e = max(e, fx_key(v[k]));
+            }
+        emax_sh[w][lane] = e;
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < kStateWarps; ++q)
+            E = max(E, emax_sh[q][lane]);
+        // pass 2: the exact total (the partials are still in L2)
+        unsigned long long s = 0;
+        if (j < D)
+            for (int b0 = w; b0 < src.nparts; b0 += kBatch * kStateWarps) {
+                float v[kBatch];
+#pragma unroll
+                for (int k = 0; k < kBatch; ++k) {
+                    const int b = b0 + k * kStateWarps;
+                    v[k] = (b < src.nparts) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+                }
+#pragma unroll
+                for (int k = 0; k < kBatch; ++k)
+                    s += fx_of(v[k], E);
+            }
+        ssum_sh[w][lane] = s;
+        __syncthreads();
+        if (w == 0)
+#pragma unroll
+            for (int q = 0; q < kStateWarps; ++q)
+                S += ssum_sh[q][lane];
+    } else if (w == 0 && j < D) {
+        S = src.sums[j];
+        E = src.scales[j];
+    }
+    if (w == 0) {
+        float cn = 0.f;
+        if (j < D) {
+            const float m = fx_value(S, E) * kc.inv_V;
+            cn = ema_pair(kc.ema, __ldcg(c + j), m);
+            c[j] = cn;
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1)
+            cn += __shfl_xor_sync(0xffffffffu, cn, o);
+        if (lane == 0)
+            csum_part[group] = cn;
+    }
+    __syncthreads();  // the shared buffers are reused by the next group
+}
+
+// Exact fixed-point total of n fp32 values load(0) .. load(n-1) (>= 0), by a
+// whole CTA of kStateThreads threads; every thread gets the result.  The
+// loader reads global memory through L2 (the values were written by other
+// CTAs) or another CTA's shared memory in a cluster.
+template <typename Load>
+__device__ float block_fx_total(Load load, int n)
+{
+    __shared__ unsigned ek[kStateWarps];
+    __shared__ unsigned long long ss[kStateWarps];
+    const int lane = threadIdx.x & 31;
+    const int w = threadIdx.x >> 5;
+    unsigned e = 0;
+    for (int b = threadIdx.x; b < n; b += kStateThreads)
+        e = max(e, fx_key(load(b)));
+    e = __reduce_max_sync(0xffffffffu, e);
+    if (lane == 0)
+        ek[w] = e;
+    __syncthreads();
+    unsigned E = 0;
+#pragma unroll
+    for (int q = 0; q < kStateWarps; ++q)
+        E = max(E, ek[q]);
+    unsigned long long s = 0;
+    for (int b = threadIdx.x; b < n; b += kStateThreads)
+        s += fx_of(load(b), E);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        s += shfl_xor_u64(s, o);
+    if (lane == 0)
+        ss[w] = s;
+    __syncthreads();
+    unsigned long long S = 0;
+#pragma unroll
+    for (int q = 0; q < kStateWarps; ++q)
+        S += ss[q];
+    __syncthreads();
+    return fx_value(S, E);
+}
+
+// The normaliser from the total of r (r_total, over the whole table) and the
+// per-group sums of the new c (load(q), q < ngroups), by a whole CTA; every
+// thread gets it.  The group sums are added in a fixed order (thread t takes
+// groups t, t + 256, ... in order, then a fixed butterfly, then the warps in
+// order), so every CTA that runs this forms the same bits.
+struct Norm {
+    float s, rbar, cbar, inv_s;
+};
+template <typename Load>
+__device__ Norm normaliser(float r_total, Load load, int ngroups, const StepConsts &kc)
+{
+    __shared__ float part[kStateWarps];
+    const int lane = threadIdx.x & 31;
+    const int w = threadIdx.x >> 5;
+    float csum = 0.f;
+    for (int q = threadIdx.x; q < ngroups; q += kStateThreads)
+        csum += load(q);
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1)
+        csum += __shfl_xor_sync(0xffffffffu, csum, o);
+    if (lane == 0)
+        part[w] = csum;
+    __syncthreads();
+    csum = 0.f;
+    for (int q = 0; q < kStateWarps; ++q)
+        csum += part[q];
+    __syncthreads();
+    Norm n;
+    n.rbar = (r_total * kc.inv_bc) * kc.inv_V;
+    n.cbar = (csum * kc.inv_bc) * kc.inv_D;
+    // the square roots taken apart: their product stays in range where
+    // rbar * cbar would underflow
+    n.s = sqrtf(n.rbar) * sqrtf(n.cbar);
+    n.inv_s = (n.s > 0.f) ? 1.f / n.s : 0.f;
+    return n;
+}
+
+// ---------------------------------------------------------------------------
+// Kernels of the three-launch form.
+// ---------------------------------------------------------------------------
+template <int VEC, int CPT, int R, bool STAGE>
+__global__ void __launch_bounds__(kThreads, kCtasPerSm)
+k_reduce_dense(const float *__restrict__ G, float *__restrict__ r, float *__restrict__ colpart,
+               float *__restrict__ rsum_part, int64_t V, int D, int ld, int tpr, StepConsts kc,
+               float *__restrict__ G_stage, float *__restrict__ rowpart, RowSpan span)
+{
+    grid_dep_wait();    // the first kernel of a step: returns at once
+    grid_dep_launch();  // the state pass may start launching now; it waits for this grid
+    extern __shared__ float comb_sh[];  // D floats: the row groups' column sums combined
+    reduce_rows<VEC, CPT, R, STAGE>(G, r, colpart + (int64_t)blockIdx.x * ld, rsum_part + blockIdx.x, V, D, ld,
+                                    tpr, kc, G_stage, rowpart, span, blockIdx.x, comb_sh,
+                                    nullptr);
+}
+
+// Column EMA and normaliser.  The first ngroups CTAs each own one group of
+// 32 columns (column_group).  For the sparse and LM-head steps and a dense
+// step in column panels the remaining CTAs also do the row pass: r for every
+// row (rows outside a sparse batch see a zero gradient row, touched rows take
+// their sum of g^2 per column slice from `rowpart`) and the sum of the new r
+// per CTA.  The last CTA to finish forms mean(rhat), mean(chat) and s; the
+// sum of r over the table is the exact fixed-point total of the nrsum per-CTA
+// sums, or, in a row-sharded step, comes with the exchanged totals.
 struct RowPass {
     float *r;               // r[V], updated (sparse step only)
     int32_t *slot;          // touched-row map, cleared here
@@ -267,73 +566,31 @@ struct RowPass {
 };
 
 __global__ void __launch_bounds__(kStateThreads)
-k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict__ rsum_part,
-              int nrsum, float *__restrict__ c, double *__restrict__ csum_part, DevScalars *sc,
-              int64_t V, int D, double beta2, double one_minus_beta2, double inv_bc, RowPass rowp)
+k_state_dense(ColSource src, float *__restrict__ rsum_part, int nrsum, float *__restrict__ c,
+              float *__restrict__ csum_part, DevScalars *sc, int64_t V, int D, StepConsts kc, RowPass rowp)
 {
-    constexpr int kW = kStateThreads / 32;
+    constexpr int kW = kStateWarps;
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
-    const int nstate = (int)gridDim.x - rowp.nrow_ctas;
-    __shared__ float part[kW][32];
-    __shared__ double part_last[kW][2];
+    const int ngroups = (int)gridDim.x - rowp.nrow_ctas;
+    __shared__ float part[kW];
     __shared__ bool am_last;
-    // GB300 runs fp64 at a small fraction of its fp32 rate, and a single
-    // fp64 pipe op per row or column showed up in this kernel's time: the
-    // per-CTA work is fp32 (the EMAs with float-pair coefficients, sums of
-    // at most a few thousand values per CTA in fixed trees), and only the
-    // sums across CTAs and the normaliser run in fp64.
-    const double inv_D = 1.0 / (double)D, inv_V = 1.0 / (double)V;
-    const EmaPair ema = make_ema_pair(beta2, one_minus_beta2);
+    // GB300 runs fp64 at a small fraction of its fp32 rate: everything here
+    // is fp32 (the EMAs with float-pair coefficients, sums of at most a few
+    // thousand values per CTA in fixed trees, the normaliser) or integer
+    // (the fixed-point totals).
     grid_dep_wait();  // column partials and row sums of the earlier passes
     grid_dep_launch();
 
-    if ((int)blockIdx.x < nstate) {
-        const int j = blockIdx.x * kStateCols + lane;
-        // rows w, w + 8, w + 16, ...: 32 loads in flight, summed pairwise
-        // within the batch, then across batches and warps in order
-        constexpr int kBatch = 32;
-        float acc = 0.f;
-        if (j < D)
-            for (int b0 = w; b0 < nparts; b0 += kBatch * kW) {
-                float v[kBatch];
-#pragma unroll
-                for (int k = 0; k < kBatch; ++k) {
-                    const int b = b0 + k * kW;
-                    v[k] = (b < nparts) ? __ldcg(colpart + (int64_t)b * D + j) : 0.f;
-                }
-#pragma unroll
-                for (int h = kBatch / 2; h >= 1; h >>= 1)
-#pragma unroll
-                    for (int k = 0; k < h; ++k)
-                        v[k] += v[k + h];
-                acc += v[0];
-            }
-        part[w][lane] = acc;
-        __syncthreads();
-        if (w == 0) {
-            float tot = 0.f;
-#pragma unroll
-            for (int q = 0; q < kW; ++q)
-                tot += part[q][lane];
-            float cn = 0.f;
-            if (j < D) {
-                const float cnew = ema_pair(ema, c[j], tot * (float)inv_V);
-                c[j] = cnew;
-                cn = cnew;
-            }
-#pragma unroll
-            for (int o = 16; o >= 1; o >>= 1)
-                cn += __shfl_xor_sync(0xffffffffu, cn, o);
-            if (lane == 0)
-                csum_part[blockIdx.x] = (double)cn;
-        }
+    if ((int)blockIdx.x < ngroups) {
+        column_group(src, blockIdx.x, c, csum_part, D, kc);
     } else {
-        const int rb = (int)blockIdx.x - nstate;
+        const int rb = (int)blockIdx.x - ngroups;
         const int64_t stride = (int64_t)rowp.nrow_ctas * kStateThreads;
         // Every row of the table: the row EMA (ema_pair), then the CTA's sum
         // of the new r in fp32 (thread, warp butterfly, warps in order).
-        const float inv_Df = (float)inv_D;
+        const float inv_Df = kc.inv_D;
+        const EmaPair &ema = kc.ema;
         float rsum = 0.f;
         if (rowp.slot == nullptr) {
             // every row: per-column-block sums, slice-major, in block order
@@ -387,13 +644,13 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
         for (int o = 16; o >= 1; o >>= 1)
             rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
         if (lane == 0)
-            part[w][0] = rsum;
+            part[w] = rsum;
         __syncthreads();
         if (threadIdx.x == 0) {
             float t = 0.f;
             for (int q = 0; q < kW; ++q)
-                t += part[q][0];
-            rsum_part[rb] = (double)t;
+                t += part[q];
+            rsum_part[rb] = t;
         }
     }
     if (threadIdx.x == 0) {
@@ -405,132 +662,253 @@ k_state_dense(const float *__restrict__ colpart, int nparts, double *__restrict_
     if (!am_last)
         return;
     __threadfence();
-    // The last CTA: thread t sums entries t, t + 256, ... in order (all its
-    // loads in flight at once), then a fixed butterfly per warp and the
-    // warps in order.
-    double csum = 0.0, rsum = 0.0;
-    for (int b = threadIdx.x; b < nstate; b += kStateThreads)
-        csum += __ldcg(csum_part + b);
-    for (int b = threadIdx.x; b < nrsum; b += kStateThreads)
-        rsum += __ldcg(rsum_part + b);
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-        csum += __shfl_xor_sync(0xffffffffu, csum, o);
-        rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
-    }
-    if (lane == 0) {
-        part_last[w][0] = csum;
-        part_last[w][1] = rsum;
-    }
-    __syncthreads();
+    const float r_total = (src.sums != nullptr)
+                              ? fx_value(src.sums[D], src.scales[D])
+                              : block_fx_total([&](int b) { return __ldcg(rsum_part + b); }, nrsum);
+    const Norm n = normaliser(r_total, [&](int q) { return __ldcg(csum_part + q); }, ngroups, kc);
     if (threadIdx.x == 0) {
-        csum = 0.0;
-        rsum = 0.0;
-        for (int q = 0; q < kW; ++q) {
-            csum += part_last[q][0];
-            rsum += part_last[q][1];
-        }
-        const double rbar = rsum * inv_bc * inv_V;
-        const double cbar = csum * inv_bc * inv_D;
-        const double s = sqrt(rbar * cbar);
-        sc->s = s;
-        sc->rbar = rbar;
-        sc->cbar = cbar;
-        sc->inv_s = (s > 0.0) ? (float)(1.0 / s) : 0.f;
+        sc->s = n.s;
+        sc->rbar = n.rbar;
+        sc->cbar = n.cbar;
+        sc->inv_s = n.inv_s;
         sc->ticket = 0u;
     }
 }
 
-// Pass 3: the update.  Same row ranges and column mapping as pass 1; each
-// CTA walks its rows from the last iteration block to the first.  The
-// column scales live in shared memory (D floats).  D columns from row stride
-// ld, as in pass 1: W, G and c point at the first column of the panel.
 template <int VEC, int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__restrict__ r,
-              const float *__restrict__ c, const DevScalars *__restrict__ sc,
-              int64_t V, int D, int ld, int tpr, float inv_bc, float eps, float lr_signed, int variant,
-              RowSpan span)
+              const float *__restrict__ c, const DevScalars *__restrict__ sc, int64_t V, int D, int ld, int tpr,
+              float inv_bc, float eps, float lr_signed, int variant, RowSpan span)
 {
-    using F = typename Vec<VEC>::F;
-    using WT = typename WRaw<BF16, VEC>::T;
-    extern __shared__ float cs[];  // D column scales
-    const int DV = D / VEC;
-    const int tid = threadIdx.x;
-    const int rg = kThreads / tpr;
-    const int g = tid / tpr;
-    const int l = tid - g * tpr;
-    const int64_t row0 = (int64_t)(span.cta_base + blockIdx.x) * V / span.nparts;
-    const int64_t row1 = (int64_t)(span.cta_base + blockIdx.x + 1) * V / span.nparts;
-    const int64_t step = (int64_t)rg * R;
-    const int64_t nblocks = (row1 - row0 + step - 1) / step;
-
     // While the state pass finishes: pull this thread's first rows of G and
     // W (the last iteration block, walked first) towards L2.
-    if (nblocks > 0) {
-        const int64_t base = row0 + (nblocks - 1) * step;
-        for (int k = 0; k < R; ++k) {
-            const int64_t i = base + (int64_t)g * R + k;
-            for (int cc = 0; cc < CPT; ++cc) {
-                const int col = l + cc * tpr;
-                if (i < row1 && col < DV) {
-                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(G + idx));
-                    asm volatile("prefetch.global.L2 [%0];" ::"l"(static_cast<const char *>(W) +
-                                                                   idx * (BF16 ? 2 : 4)));
+    {
+        const int rg = kThreads / tpr;
+        const int g = threadIdx.x / tpr;
+        const int l = threadIdx.x - g * tpr;
+        const int DV = D / VEC;
+        const int64_t row0 = (int64_t)(span.cta_base + blockIdx.x) * V / span.nparts;
+        const int64_t row1 = (int64_t)(span.cta_base + blockIdx.x + 1) * V / span.nparts;
+        const int64_t step = (int64_t)rg * R;
+        const int64_t nblocks = (row1 - row0 + step - 1) / step;
+        if (nblocks > 0) {
+            const int64_t base = row0 + (nblocks - 1) * step;
+            for (int k = 0; k < R; ++k) {
+                const int64_t i = base + (int64_t)g * R + k;
+                for (int cc = 0; cc < CPT; ++cc) {
+                    const int col = l + cc * tpr;
+                    if (i < row1 && col < DV) {
+                        const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(G + idx));
+                        asm volatile("prefetch.global.L2 [%0];" ::"l"(static_cast<const char *>(W) +
+                                                                       idx * (BF16 ? 2 : 4)));
+                    }
                 }
             }
         }
     }
     grid_dep_wait();  // c, s (state pass) and r (reduce pass)
     grid_dep_launch();
+    apply_rows<VEC, CPT, R, BF16>(W, G, r, c, __ldcg(&sc->inv_s), V, D, ld, tpr, inv_bc, eps, lr_signed, variant,
+                                  span, blockIdx.x);
+}
 
-    // column scale sqrt(chat_j / s) (FULL), sqrt(chat_j) (COL) or 1 (ROW)
-    const float inv_s = (variant == EMBER_VARIANT_FULL) ? sc->inv_s : 1.f;
-    for (int j = tid; j < D; j += kThreads)
-        cs[j] = (variant == EMBER_VARIANT_ROW) ? 1.f : sqrtf(c[j] * inv_bc * inv_s);
-    __syncthreads();
+// ---------------------------------------------------------------------------
+// Small tables in one launch: one thread-block cluster of nparts <= 8 CTAs
+// (the same CTA grid and row ranges as the three-launch form).  Each CTA
+//   - starts copying its rows of W into shared memory (cp.async) and loads
+//     the old c;
+//   - reduces its rows with reduce_rows, keeping every element of G it loads
+//     in a thread-private slot of shared memory, and leaves its column
+//     partial and its sum of r in its own shared memory;
+//   - cluster barrier; then reads every CTA's partials through distributed
+//     shared memory and forms, for ALL columns, the column totals, the new c
+//     and the normaliser itself (the same integer totals, EMA and fixed
+//     summation order as column_group / block_fx_total / normaliser, hence
+//     the same bits as the three-launch form);
+//   - updates its rows from the kept G and W.
+// G is read from HBM once (4VD + 2wVD bytes in all, not 8VD + 2wVD), and the
+// only synchronisation is the cluster's hardware barrier, so the step is a
+// single short launch.  Used when the kept G and W fit shared memory.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ void cluster_barrier()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
-    for (int64_t b = nblocks - 1; b >= 0; --b) {
-        const int64_t base = row0 + b * step;
-        F gv[R][CPT];
-        WT wr[R][CPT];
+// A float of CTA `rank`'s shared memory at the address `local` has in this CTA.
+__device__ __forceinline__ float ld_dsmem(const float *local, unsigned rank)
+{
+    uint32_t a = (uint32_t)__cvta_generic_to_shared(local), ra;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(ra) : "r"(a), "r"(rank));
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(ra) : "memory");
+    return v;
+}
+
+struct SmallArgs {
+    void *W;
+    const float *G;
+    float *r, *c;
+    DevScalars *sc;
+    int64_t V;
+    int D, tpr, nits;
+    StepConsts kc;
+    float eps, lr_signed;
+    int variant;
+};
+
+constexpr int kMaxClusterCtas = 8;
+constexpr size_t kSmallSmemMax = 200 << 10;
+
+// Shared memory of k_dense_cluster, in bytes from the dynamic base: kept G,
+// kept W, then D floats each of the column partial, the combine buffer, the
+// old c, the new c (then the column scales), and ceil(D/32) floats.
+template <int CPT, int R, bool BF16>
+__host__ __device__ constexpr size_t small_slots(int nits) { return (size_t)nits * R * CPT * kThreads; }
+template <int CPT, int R, bool BF16>
+__host__ __device__ constexpr size_t small_smem_bytes(int nits, int D)
+{
+    return small_slots<CPT, R, BF16>(nits) * (16 + (BF16 ? 8 : 16)) + (size_t)4 * D * sizeof(float) +
+           (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float);
+}
+
+template <int CPT, int R, bool BF16>
+__global__ void __launch_bounds__(kThreads, 1)
+k_dense_cluster(SmallArgs a)
+{
+    constexpr int VEC = 4;
+    using F = float4;
+    using WT = typename WRaw<BF16, VEC>::T;
+    extern __shared__ __align__(16) unsigned char sm_dyn[];
+    const size_t nslot = small_slots<CPT, R, BF16>(a.nits);
+    F *keepG = reinterpret_cast<F *>(sm_dyn);
+    WT *keepW = reinterpret_cast<WT *>(sm_dyn + nslot * 16);
+    float *cpart = reinterpret_cast<float *>(sm_dyn + nslot * (16 + sizeof(WT)));
+    float *comb = cpart + a.D;
+    float *cold = comb + a.D;
+    float *cnew = cold + a.D;
+    float *csum_sh = cnew + a.D;
+    __shared__ float rsum_own;
+
+    const int D = a.D, DV = D / VEC, tid = threadIdx.x;
+    const int tpr = a.tpr, rg = kThreads / tpr, g = tid / tpr, l = tid - g * tpr;
+    const unsigned nb = gridDim.x;
+    const unsigned cta = blockIdx.x;  // the grid is one cluster: the rank in it
+    const RowSpan span{0, (int)nb, 0};
+    const int64_t row0 = (int64_t)cta * a.V / nb, row1 = (int64_t)(cta + 1) * a.V / nb;
+    const int rows_per_it = rg * R;
+
+    // this CTA's rows of W into its slots, while G is reduced
+    for (int it = 0; it < a.nits; ++it)
 #pragma unroll
         for (int k = 0; k < R; ++k) {
-            const int64_t i = base + (int64_t)g * R + k;
+            const int64_t i = row0 + (int64_t)it * rows_per_it + (int64_t)g * R + k;
 #pragma unroll
-            for (int cc = 0; cc < CPT; ++cc) {
-                const int col = l + cc * tpr;
+            for (int c = 0; c < CPT; ++c) {
+                const int col = l + c * tpr;
                 if (i < row1 && col < DV) {
-                    const int64_t idx = (i - span.row_base) * ld + (int64_t)col * VEC;
-                    gv[k][cc] = load_g<VEC>(G + idx);
-                    wr[k][cc] = load_w<BF16, VEC>(W, idx);
+                    WT *dst = keepW + ((it * R + k) * CPT + c) * kThreads + tid;
+                    const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst);
+                    if constexpr (BF16)
+                        asm volatile("cp.async.ca.shared.global [%0], [%1], 8;" ::"r"(d),
+                                     "l"(static_cast<const unsigned short *>(a.W) + i * D + (int64_t)col * VEC)
+                                     : "memory");
+                    else
+                        asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(d),
+                                     "l"(static_cast<const float *>(a.W) + i * D + (int64_t)col * VEC)
+                                     : "memory");
                 }
             }
         }
+    asm volatile("cp.async.commit_group;" ::: "memory");
+    for (int j = tid; j < D; j += kThreads)
+        cold[j] = a.c[j];
+
+    reduce_rows<VEC, CPT, R, false, true>(a.G, a.r, cpart, &rsum_own, a.V, D, D, tpr, a.kc, nullptr, nullptr, span,
+                                          cta, comb, keepG);
+    cluster_barrier();  // every CTA's partials are in its shared memory
+
+    // the column pass for every column, as column_group forms it
+    const int lane = tid & 31, w = tid >> 5;
+    const int ngroups = (D + kStateCols - 1) / kStateCols;
+    for (int q = w; q < ngroups; q += kStateWarps) {
+        const int j = q * kStateCols + lane;
+        float v[kMaxClusterCtas];
+        unsigned E = 0;
 #pragma unroll
-        for (int k = 0; k < R; ++k) {
-            const int64_t i = base + (int64_t)g * R + k;
-            if (i >= row1)
-                continue;
-            const float rs = (variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(__ldg(r + i) * inv_bc);
+        for (int b = 0; b < kMaxClusterCtas; ++b) {
+            v[b] = (b < (int)nb && j < D) ? ld_dsmem(cpart + j, b) : 0.f;
+            E = max(E, fx_key(v[b]));
+        }
+        unsigned long long S = 0;
 #pragma unroll
-            for (int cc = 0; cc < CPT; ++cc) {
-                const int col = l + cc * tpr;
-                if (col >= DV)
-                    continue;
-                float w[VEC];
-                unpack_w(wr[k][cc], w);
+        for (int b = 0; b < kMaxClusterCtas; ++b)
+            S += fx_of(v[b], E);
+        float cn = 0.f;
+        if (j < D) {
+            const float m = fx_value(S, E) * a.kc.inv_V;
+            cn = ema_pair(a.kc.ema, cold[j], m);
+            cnew[j] = cn;
+        }
 #pragma unroll
-                for (int e = 0; e < VEC; ++e) {
-                    const float den = fmaf(rs, cs[col * VEC + e], eps);
-                    const float u = comp(gv[k][cc], e) / den;
-                    w[e] = fmaf(lr_signed, u, w[e]);
-                }
-                store_w<BF16, VEC>(W, (i - span.row_base) * ld + (int64_t)col * VEC, w);
-            }
+        for (int o = 16; o >= 1; o >>= 1)
+            cn += __shfl_xor_sync(0xffffffffu, cn, o);
+        if (lane == 0)
+            csum_sh[q] = cn;
+    }
+    const float r_total = block_fx_total([&](int b) { return ld_dsmem(&rsum_own, b); }, (int)nb);
+    cluster_arrive();  // done reading the other CTAs' shared memory
+    const Norm n = normaliser(r_total, [&](int q) { return csum_sh[q]; }, ngroups, a.kc);
+    if (cta == 0) {
+        for (int j = tid; j < D; j += kThreads)
+            a.c[j] = cnew[j];
+        if (tid == 0) {
+            a.sc->s = n.s;
+            a.sc->rbar = n.rbar;
+            a.sc->cbar = n.cbar;
+            a.sc->inv_s = n.inv_s;
         }
     }
+
+    // the update, as apply_rows forms it, from the kept G and W
+    const float inv_bc = a.kc.inv_bc;
+    const float inv_s = (a.variant == EMBER_VARIANT_FULL) ? n.inv_s : 1.f;
+    float *cs = cnew;  // the column scales replace the new c (already written out)
+    __syncthreads();
+    for (int j = tid; j < D; j += kThreads)
+        cs[j] = (a.variant == EMBER_VARIANT_ROW) ? 1.f : sqrtf(cnew[j] * inv_bc * inv_s);
+    asm volatile("cp.async.wait_all;" ::: "memory");
+    __syncthreads();
+    for (int it = 0; it < a.nits; ++it)
+#pragma unroll
+        for (int k = 0; k < R; ++k) {
+            const int64_t i = row0 + (int64_t)it * rows_per_it + (int64_t)g * R + k;
+            if (i >= row1)
+                continue;
+            const float rs = (a.variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(__ldcg(a.r + i) * inv_bc);
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col = l + c * tpr;
+                if (col >= DV)
+                    continue;
+                const int slot = ((it * R + k) * CPT + c) * kThreads + tid;
+                const F gv = keepG[slot];
+                float wv[VEC];
+                unpack_w(keepW[slot], wv);
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {
+                    const float den = fmaf(rs, cs[col * VEC + e], a.eps);
+                    const float u = comp(gv, e) / den;
+                    wv[e] = fmaf(a.lr_signed, u, wv[e]);
+                }
+                store_w<BF16, VEC>(a.W, i * D + (int64_t)col * VEC, wv);
+            }
+        }
+    cluster_wait();  // no CTA leaves while another may still read its shared memory
 }
 
 // Row-only Ember in one pass (variant ROW: vtil_ij = rhat_i, the "row-only"
@@ -567,8 +945,8 @@ __device__ __forceinline__ void cp_async_wait_prev() { asm volatile("cp.async.wa
 template <int VEC, int CPT, int R, bool BF16, bool ASYNC>
 __global__ void __launch_bounds__(kThreads, kCtasPerSm)
 k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__restrict__ r,
-                float *__restrict__ colpart, double *__restrict__ rsum_part, int64_t V, int D, int tpr,
-                double beta2, double one_minus_beta2, float inv_bc, float eps, float lr_signed)
+                float *__restrict__ colpart, float *__restrict__ rsum_part, int64_t V, int D, int tpr,
+                StepConsts kc, float eps, float lr_signed)
 {
     static_assert(!ASYNC || VEC == 4, "the staged copies move 16-byte slices");
     using F = typename Vec<VEC>::F;
@@ -586,7 +964,7 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
     const int64_t row1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
     __shared__ float red[kWarps][R];
     __shared__ float rs_sh[kThreads / 32 * R];  // sqrt(rhat) of this iteration's rows
-    __shared__ double rsum_sh[kWarps];
+    __shared__ float rsum_sh[kWarps];
     // ASYNC: two stages of [R][CPT][kThreads] slices of G, then of W; the
     // column-sum combine buffer (D floats) follows
     extern __shared__ __align__(16) unsigned char ro_dyn[];
@@ -631,7 +1009,7 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
             acc[c][e] = 0.f;
-    double rsum = 0.0;
+    float rsum = 0.f;
     const int rows_per_it = rg * R;
     for (int64_t base = row0; base < row1; base += rows_per_it) {
         F v[R][CPT];
@@ -689,11 +1067,10 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
                 float sum = 0.f;
                 for (int q = 0; q < wpg; ++q)
                     sum += red[g * wpg + q][l];
-                const double mean_row = (double)sum / (double)D;
-                const float rn = (float)(beta2 * (double)r[i] + one_minus_beta2 * mean_row);
+                const float rn = ema_pair(kc.ema, r[i], sum * kc.inv_D);
                 r[i] = rn;
-                rsum += (double)rn;
-                rsv = sqrtf(rn * inv_bc);
+                rsum += rn;
+                rsv = sqrtf(rn * kc.inv_bc);
             }
             rs_sh[g * R + l] = rsv;
         }
@@ -755,32 +1132,47 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
         rsum_sh[warp] = rsum;
     __syncthreads();
     if (tid == 0) {
-        double t = 0.0;
+        float t = 0.f;
         for (int q = 0; q < kWarps; ++q)
             t += rsum_sh[q];
         rsum_part[blockIdx.x] = t;
     }
 }
 
-// Row-sharded step: copy the per-CTA partials of every shard's exchange
-// block (CTA b is entry b % cap of shard b / cap) into the workspace layout
-// of the whole-table step, in CTA order.
-__global__ void k_shard_unpack(const unsigned char *__restrict__ blocks, size_t block_bytes, size_t block_rsum,
-                               int cap, int nparts, int D, float *__restrict__ colpart,
-                               double *__restrict__ rsum_part)
+// ---------------------------------------------------------------------------
+// Row-sharded step, phases 1 and 2 (after the shard's reduce launch, whose
+// ncta partial rows sit in the shard's workspace).
+//   k_shard_scales: per column (and, at index D, for the per-CTA sums of r)
+//       the largest key among the shard's partials -> scales[0..D].
+//   k_shard_pack: per column the fixed-point sum of the shard's partials at
+//       the all-reduced scales -> sums[0..D].
+// One thread per column; the partial rows are read with coalesced loads.
+// ---------------------------------------------------------------------------
+__global__ void k_shard_scales(const float *__restrict__ colpart, const float *__restrict__ rsum_part, int ncta,
+                               int D, unsigned char *__restrict__ scales)
 {
     grid_dep_wait();
     grid_dep_launch();
-    const int64_t total = (int64_t)nparts * D;
-    for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < total;
-         q += (int64_t)gridDim.x * blockDim.x) {
-        const int b = (int)(q / D);
-        const int j = (int)(q - (int64_t)b * D);
-        const float *src = reinterpret_cast<const float *>(blocks + (size_t)(b / cap) * block_bytes);
-        colpart[q] = src[(int64_t)(b % cap) * D + j];
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= D; j += gridDim.x * blockDim.x) {
+        unsigned e = 0;
+        for (int b = 0; b < ncta; ++b)
+            e = max(e, fx_key(j < D ? __ldcg(colpart + (int64_t)b * D + j) : __ldcg(rsum_part + b)));
+        scales[j] = (unsigned char)e;
     }
-    for (int b = blockIdx.x * blockDim.x + threadIdx.x; b < nparts; b += gridDim.x * blockDim.x)
-        rsum_part[b] = reinterpret_cast<const double *>(blocks + (size_t)(b / cap) * block_bytes + block_rsum)[b % cap];
+}
+
+__global__ void k_shard_pack(const float *__restrict__ colpart, const float *__restrict__ rsum_part, int ncta,
+                             int D, const unsigned char *__restrict__ scales, unsigned long long *__restrict__ sums)
+{
+    grid_dep_wait();
+    grid_dep_launch();
+    for (int j = blockIdx.x * blockDim.x + threadIdx.x; j <= D; j += gridDim.x * blockDim.x) {
+        const unsigned E = scales[j];
+        unsigned long long s = 0;
+        for (int b = 0; b < ncta; ++b)
+            s += fx_of(j < D ? __ldcg(colpart + (int64_t)b * D + j) : __ldcg(rsum_part + b), E);
+        sums[j] = s;
+    }
 }
 
 template <int VEC, int CPT>
@@ -788,11 +1180,12 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 {
     constexpr int R1 = (16 / CPT) < 1 ? 1 : (16 / CPT);
     constexpr int R3 = (8 / CPT) < 1 ? 1 : (8 / CPT);
-    const int nparts = dense_parts(a.V);
+    const int nparts = dense_parts(a.V, a.D);
     const int D = (int)a.D;
     DevScalars *sc = reinterpret_cast<DevScalars *>(a.ws + a.lay.scalars);
-    double *rsum_part = reinterpret_cast<double *>(a.ws + a.lay.rsum_part);
-    double *csum_part = reinterpret_cast<double *>(a.ws + a.lay.csum_part);
+    float *rsum_part = reinterpret_cast<float *>(a.ws + a.lay.rsum_part);
+    float *csum_part = reinterpret_cast<float *>(a.ws + a.lay.csum_part);
+    const StepConsts kc = make_consts(a.beta2, a.one_minus_beta2, a.V, a.D, a.inv_bc);
     float *colpart = reinterpret_cast<float *>(a.ws + a.lay.colpart);
     const int rg = kThreads / a.map.tpr;
     // column panels (one unless D is wider than a CTA's row): columns
@@ -817,33 +1210,39 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             return cudaErrorInvalidValue;  // refused by the entry points
         const int ncta = sh.cta_end - sh.cta_begin;
         span = RowSpan{sh.cta_begin, nparts, sh.row_base};
+        const int nthr = 256;
+        const int nblk = (D + 1 + nthr - 1) / nthr;
         if (sh.phase == 1) {
-            if (ncta == 0)
-                return cudaSuccess;
-            float *bcol = static_cast<float *>(sh.block);
-            double *brsum = reinterpret_cast<double *>(static_cast<unsigned char *>(sh.block) + sh.block_rsum);
-            e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(ncta), dim3(kThreads), shmem, a.stream, false,
-                         a.G, a.r, bcol, brsum, a.V, D, ld, a.map.tpr, a.beta2, a.one_minus_beta2, nullptr,
-                         nullptr, span);
+            if (ncta > 0) {
+                e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(ncta), dim3(kThreads), shmem, a.stream, false,
+                             a.G, a.r, colpart, rsum_part, a.V, D, ld, a.map.tpr, kc,
+                             nullptr, nullptr, span);
+                if (e != cudaSuccess)
+                    return e;
+            }
+            e = launch_k(k_shard_scales, dim3(nblk), dim3(nthr), 0, a.stream, false, colpart, rsum_part, ncta, D,
+                         sh.scales);
             return e != cudaSuccess ? e : cudaGetLastError();
         }
-        e = launch_k(k_shard_unpack, dim3(kGridCtas), dim3(kThreads), 0, a.stream, false,
-                     static_cast<const unsigned char *>(sh.blocks), sh.block_bytes, sh.block_rsum, sh.cap, nparts, D,
-                     colpart, rsum_part);
-        if (e != cudaSuccess)
-            return e;
-        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        if (sh.phase == 2) {
+            e = launch_k(k_shard_pack, dim3(nblk), dim3(nthr), 0, a.stream, false, colpart, rsum_part, ncta, D,
+                         sh.scales, sh.sums);
+            return e != cudaSuccess ? e : cudaGetLastError();
+        }
+        const ColSource src{nullptr, 0, sh.sums, sh.scales};
+        e = launch_k(k_state_dense, dim3((D + kStateCols - 1) / kStateCols), dim3(kStateThreads), 0, a.stream,
+                     false, src, rsum_part, 0, a.c, csum_part, sc, a.V, D, kc,
+                     RowPass{nullptr, nullptr, nullptr, 0, 0});
         if (e != cudaSuccess || ncta == 0)
             return e != cudaSuccess ? e : cudaGetLastError();
         const size_t cs_bytes = (size_t)D * sizeof(float);
         if (a.wbf16)
             e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
-                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, kc.inv_bc, a.eps, a.lr_signed,
                          a.variant, span);
         else
             e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(ncta), dim3(kThreads), cs_bytes, a.stream, pdl,
-                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, (float)a.inv_bc, a.eps, a.lr_signed,
+                         a.W, a.G, a.r, a.c, sc, a.V, D, ld, a.map.tpr, kc.inv_bc, a.eps, a.lr_signed,
                          a.variant, span);
         return e != cudaSuccess ? e : cudaGetLastError();
     }
@@ -859,7 +1258,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
             if (e == cudaSuccess)
                 e = launch_k(k, dim3(nparts), dim3(kThreads), sm, a.stream, false, a.W, a.G, a.r, colpart,
-                             rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, (float)a.inv_bc, a.eps,
+                             rsum_part, a.V, D, a.map.tpr, kc, a.eps,
                              a.lr_signed);
         } else {
             auto *k = k_rowonly_dense<VEC, CPT, RR, false, kAsync>;
@@ -867,15 +1266,14 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
             if (e == cudaSuccess)
                 e = launch_k(k, dim3(nparts), dim3(kThreads), sm, a.stream, false, a.W, a.G, a.r, colpart,
-                             rsum_part, a.V, D, a.map.tpr, a.beta2, a.one_minus_beta2, (float)a.inv_bc, a.eps,
+                             rsum_part, a.V, D, a.map.tpr, kc, a.eps,
                              a.lr_signed);
         }
         if (e != cudaSuccess)
             return e;
         if (a.trace)
             cudaEventRecord(a.trace[1], a.stream);
-        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                         a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+        e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, kc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
         if (e != cudaSuccess)
             return e;
         if (a.trace) {
@@ -883,6 +1281,38 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             cudaEventRecord(a.trace[3], a.stream);
         }
         return cudaGetLastError();
+    }
+    if constexpr (VEC == 4) {
+        if (!a.lm && !a.G_stage && !a.trace && np == 1 && nparts <= kMaxClusterCtas) {
+            // a small table: the whole step in one cluster launch, when the
+            // kept G and W fit shared memory
+            const int64_t rows = (a.V + nparts - 1) / nparts;
+            const int rows_per_it = rg * R1;
+            const int nits = (int)((rows + rows_per_it - 1) / rows_per_it);
+            const size_t sm = a.wbf16 ? small_smem_bytes<CPT, R1, true>(nits, D)
+                                      : small_smem_bytes<CPT, R1, false>(nits, D);
+            if (sm <= kSmallSmemMax) {
+                auto *k = a.wbf16 ? k_dense_cluster<CPT, R1, true> : k_dense_cluster<CPT, R1, false>;
+                e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+                if (e != cudaSuccess)
+                    return e;
+                SmallArgs sa{a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, nits, kc, a.eps, a.lr_signed, a.variant};
+                cudaLaunchConfig_t cfg = {};
+                cfg.gridDim = dim3(nparts);
+                cfg.blockDim = dim3(kThreads);
+                cfg.dynamicSmemBytes = sm;
+                cfg.stream = a.stream;
+                cudaLaunchAttribute attr[1];
+                attr[0].id = cudaLaunchAttributeClusterDimension;
+                attr[0].val.clusterDim.x = nparts;
+                attr[0].val.clusterDim.y = 1;
+                attr[0].val.clusterDim.z = 1;
+                cfg.attrs = attr;
+                cfg.numAttrs = 1;
+                e = cudaLaunchKernelEx(&cfg, k, sa);
+                return e != cudaSuccess ? e : cudaGetLastError();
+            }
+        }
     }
     if (a.lm) {
         // G comes from the LM-head kernel, which also leaves the sums of g^2
@@ -902,7 +1332,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         const int64_t vb = (a.V + kStateThreads - 1) / kStateThreads;
         const int nrow_ctas = (int)(vb < kMaxRowCtas ? vb : kMaxRowCtas);
         e = launch_state(lm_col, lmhead_row_blocks(a.V), rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D,
-                         a.beta2, a.one_minus_beta2, a.inv_bc, a.stream, false, a.r, nullptr, lm_row,
+                         kc, a.stream, false, a.r, nullptr, lm_row,
                          lmhead_col_blocks(a.D), nrow_ctas);
         if (e != cudaSuccess)
             return e;
@@ -919,24 +1349,22 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             if (a.G_stage)
                 e = launch_k(k_reduce_dense<VEC, CPT, R1, true>, dim3(nparts), dim3(kThreads), shmem, a.stream,
                              pdl && q > 0, a.G + c0, a.r, colpart + c0, rsum_part, a.V, cols(q), ld, a.map.tpr,
-                             a.beta2, a.one_minus_beta2, a.G_stage + c0, rp, span);
+                             kc, a.G_stage + c0, rp, span);
             else
                 e = launch_k(k_reduce_dense<VEC, CPT, R1, false>, dim3(nparts), dim3(kThreads), shmem, a.stream,
                              pdl && q > 0, a.G + c0, a.r, colpart + c0, rsum_part, a.V, cols(q), ld, a.map.tpr,
-                             a.beta2, a.one_minus_beta2, nullptr, rp, span);
+                             kc, nullptr, rp, span);
             if (e != cudaSuccess)
                 return e;
         }
         if (a.trace)
             cudaEventRecord(a.trace[1], a.stream);
         if (np == 1) {
-            e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, a.beta2,
-                             a.one_minus_beta2, a.inv_bc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
+            e = launch_state(colpart, nparts, rsum_part, nparts, a.c, csum_part, sc, a.V, D, kc, a.stream, pdl, nullptr, nullptr, nullptr, 0, 0);
         } else {
             const int64_t vb = (a.V + kStateThreads - 1) / kStateThreads;
             const int nrow_ctas = (int)(vb < kMaxRowCtas ? vb : kMaxRowCtas);
-            e = launch_state(colpart, nparts, rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D, a.beta2,
-                             a.one_minus_beta2, a.inv_bc, a.stream, pdl, a.r, nullptr, rowpart, np, nrow_ctas);
+            e = launch_state(colpart, nparts, rsum_part, nrow_ctas, a.c, csum_part, sc, a.V, D, kc, a.stream, pdl, a.r, nullptr, rowpart, np, nrow_ctas);
         }
         if (e != cudaSuccess)
             return e;
@@ -953,11 +1381,11 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         if (a.wbf16)
             e = launch_k(k_apply_dense<VEC, CPT, R3, true>, dim3(nparts), dim3(kThreads), cs_bytes,
                          a.stream, pdl, Wq, Gd + c0, a.r, a.c + c0, sc, a.V, cols(q), ld, a.map.tpr,
-                         (float)a.inv_bc, a.eps, a.lr_signed, a.variant, span);
+                         kc.inv_bc, a.eps, a.lr_signed, a.variant, span);
         else
             e = launch_k(k_apply_dense<VEC, CPT, R3, false>, dim3(nparts), dim3(kThreads), cs_bytes,
                          a.stream, pdl, Wq, Gd + c0, a.r, a.c + c0, sc, a.V, cols(q), ld, a.map.tpr,
-                         (float)a.inv_bc, a.eps, a.lr_signed, a.variant, span);
+                         kc.inv_bc, a.eps, a.lr_signed, a.variant, span);
         if (e != cudaSuccess)
             return e;
     }
@@ -968,15 +1396,16 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 
 }  // namespace
 
-cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, int nrsum, float *c,
-                         double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl,
-                         float *r_rows, int32_t *slot, const float *rowpart, int nslices, int nrow_ctas)
+cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
+                         float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &kc,
+                         cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
+                         int nslices, int nrow_ctas)
 {
-    const int nstate = (D + kStateCols - 1) / kStateCols;
+    const int ngroups = (D + kStateCols - 1) / kStateCols;
     RowPass rp{r_rows, slot, rowpart, nslices, nrow_ctas};
-    return launch_k(k_state_dense, dim3(nstate + nrow_ctas), dim3(kStateThreads), 0, stream, pdl, colpart,
-                    nparts, rsum_part, nrsum, c, csum_part, sc, V, D, beta2, one_minus_beta2, inv_bc, rp);
+    const ColSource src{colpart, nparts, nullptr, nullptr};
+    return launch_k(k_state_dense, dim3(ngroups + nrow_ctas), dim3(kStateThreads), 0, stream, pdl, src,
+                    rsum_part, nrsum, c, csum_part, sc, V, D, kc, rp);
 }
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)

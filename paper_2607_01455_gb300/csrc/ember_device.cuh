@@ -135,5 +135,135 @@ __device__ __forceinline__ void store_w(void *W, int64_t idx, const float (&w)[V
     }
 }
 
+__device__ __forceinline__ uint64_t now_ns()
+{
+    uint64_t t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ unsigned ld_acquire(const unsigned *p)
+{
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Grid-wide barrier for a cooperative launch (every CTA co-resident), with a
+// bounded wait.  count: arrivals at the current barrier (returned to zero
+// by the last arriver); gen: barriers completed; abort: set by a CTA whose
+// wait ran past limit_ns, after which this and every later barrier fails at
+// once.  A CTA that sees false must return without touching shared results.
+// The pattern of the CUDA programming model's grid synchronisation: the CTA
+// barrier orders the CTA's writes before thread 0's fence and arrival; the
+// waiters' acquire loads order everything after it.  *t_release (optional)
+// receives the release time from the last arriver.
+static __device__ __noinline__ bool grid_sync(unsigned *count, unsigned *gen, unsigned *abort, unsigned *flags,
+                                       unsigned timeout_bit, unsigned nblocks, uint64_t limit_ns,
+                                       unsigned long long *t_release)
+{
+    __shared__ int ok_sh;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int ok = 1;
+        const unsigned g0 = ld_acquire(gen);
+        __threadfence();
+        const unsigned arrived = atomicAdd(count, 1u) + 1u;
+        if (arrived == nblocks) {
+            atomicExch(count, 0u);
+            if (t_release)
+                *t_release = now_ns();
+            __threadfence();
+            atomicAdd(gen, 1u);
+        } else {
+            const uint64_t t0 = now_ns();
+            for (unsigned k = 1; ld_acquire(gen) == g0; ++k) {
+                if ((k & 15u) == 0) {
+                    if (ld_acquire(abort)) {
+                        ok = 0;
+                        break;
+                    }
+                    if (now_ns() - t0 > limit_ns) {
+                        atomicOr(flags, timeout_bit);
+                        atomicExch(abort, 1u);
+                        ok = 0;
+                        break;
+                    }
+                }
+            }
+        }
+        if (ok && ld_acquire(abort))
+            ok = 0;
+        __threadfence();
+        ok_sh = ok;
+    }
+    __syncthreads();
+    return ok_sh != 0;
+}
+
+// ---------------------------------------------------------------------------
+// Exact sums of non-negative fp32 values in 64-bit fixed point.
+//
+// The statistics of a step are sums over the whole table of per-CTA fp32
+// partial sums (of g^2 per column, of the new r per row block).  Adding
+// those partials as integers makes the total independent of how they are
+// grouped: the same bits whether one CTA, the state pass or an all-reduce
+// across row shards forms it.  The scale is shared by all partials of one
+// sum: E, the largest biased fp32 exponent among them, maps the largest
+// partial below 2^(24 + kFxShift) = 2^50, so that up to 4096 partials add
+// up below 2^62 without overflow.  A partial 2^k times smaller than the
+// largest loses its lowest max(0, k - 26) bits; the total is exact to
+// within 2^-41 of itself for 304 partials.  NaN or Inf partials (biased
+// exponent 255, or a sign bit) make the total NaN or Inf as a float sum
+// would.
+// ---------------------------------------------------------------------------
+constexpr int kFxShift = 26;
+constexpr unsigned kFxSpecial = 255u;
+
+// Key of p for the shared scale: its biased exponent (0 for zero and
+// subnormals), 255 for NaN, Inf or a negative value.
+__device__ __forceinline__ unsigned fx_key(float p)
+{
+    const unsigned b = __float_as_uint(p);
+    return (b >> 23) > 254u ? kFxSpecial : (b >> 23);
+}
+
+// p in units of 2^(max(E,1) - 150 - kFxShift), where E >= fx_key(p) is the
+// largest key among the values summed.  When E == 255 (some value is NaN,
+// Inf or negative) the units change meaning: NaN counts 2^32, +Inf counts 1,
+// anything else 0, so that every grouping of the same values gives the
+// same total and fx_value() tells NaN from Inf.
+__device__ __forceinline__ unsigned long long fx_of(float p, unsigned E)
+{
+    const unsigned b = __float_as_uint(p);
+    if (E >= kFxSpecial)
+        return isnan(p) ? (1ull << 32) : (b == 0x7F800000u ? 1ull : 0ull);
+    const unsigned ef = b >> 23;
+    const unsigned long long M = (b & 0x7FFFFFu) | (ef ? 0x800000u : 0u);
+    const int sh = (int)(ef ? ef : 1u) - (int)(E ? E : 1u) + kFxShift;
+    if (sh >= 0)
+        return M << sh;
+    return sh > -32 ? (M >> (unsigned)(-sh)) : 0ull;
+}
+
+// The fixed-point total S at scale exponent E as a float: S rounded to
+// fp32, then scaled by 2^(max(E,1) - 150 - kFxShift) in two exact steps (the
+// total is at least 2^(E - 127) when E >= 1, so neither step underflows
+// before the last); NaN or +Inf when E == 255.
+__device__ __forceinline__ float fx_value(unsigned long long S, unsigned E)
+{
+    if (E >= kFxSpecial)
+        return (S >> 32) ? __uint_as_float(0x7FC00000u) : __uint_as_float(0x7F800000u);
+    const float x = (float)S;  // S < 2^62
+    return (x * 0x1p-49f) * __uint_as_float((E ? E : 1u) << 23);  // 2^-49 * 2^(E-127)
+}
+
+__device__ __forceinline__ unsigned long long shfl_xor_u64(unsigned long long x, int m)
+{
+    const unsigned lo = __shfl_xor_sync(0xffffffffu, (unsigned)x, m);
+    const unsigned hi = __shfl_xor_sync(0xffffffffu, (unsigned)(x >> 32), m);
+    return ((unsigned long long)hi << 32) | lo;
+}
+
 }  // namespace dev
 }  // namespace ember

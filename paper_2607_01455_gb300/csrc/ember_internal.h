@@ -50,6 +50,11 @@ struct DevScalars {
     unsigned flags;    // sticky device error bits (kFlag*)
     int32_t n_unique;  // sparse step: number of distinct valid ids
     int32_t n_valid;   // sparse step: number of ids inside [0, V)
+    // grid barrier of kernels whose CTAs wait on one another (cooperative
+    // launches): arrivals at the current barrier, barriers completed, and a
+    // word set when a bounded wait gave up (every later barrier then fails
+    // at once until ember_get_device_status clears it)
+    unsigned bar_count, bar_gen, bar_abort, bar_pad;
 };
 
 // Sparse step: ids are sorted in tiles of kSortTile keys by kSortThreads
@@ -60,8 +65,8 @@ constexpr int kSortThreads = 256;
 // Workspace layout (byte offsets, each 256-byte aligned).
 struct Layout {
     size_t scalars;     // DevScalars
-    size_t rsum_part;   // double[kRsumParts]           sum of new r per CTA
-    size_t csum_part;   // double[ceil(D/32)]           sum of new c per state CTA
+    size_t rsum_part;   // float[kRsumParts]            sum of new r per CTA
+    size_t csum_part;   // float[ceil(D/32)]            sum of new c per 32-column group
     size_t colpart;     // float[kPartRows * D]     column sums of g^2 per CTA
     // sparse step (present when max_sparse_N > 0); N = max_sparse_N,
     // Npad = N rounded up to kSortTile
@@ -112,6 +117,7 @@ struct LmArgs {
     const void *dlogits;  // T x V bf16
     const void *hidden;   // T x D bf16
     float *G;             // V x D fp32, written
+    uint64_t wait_ns;     // limit of the kernel's main-loop waits (0: the default)
 };
 
 int lmhead_row_blocks(int64_t V);
@@ -133,18 +139,16 @@ struct RowSpan {
     int64_t row_base;
 };
 
-// Row-sharded dense step (see ember_shard_reduce / ember_shard_update).
+// Row-sharded dense step (see ember_shard_reduce / ember_shard_pack /
+// ember_shard_update).
 constexpr int kMaxShards = 4096;
 struct ShardArgs {
-    int phase;            // 1: reduce and write this shard's exchange block; 2: state and apply
-    int cta_begin, cta_end;
-    int cap;              // CTAs per shard block (the last shard may use fewer)
-    int nshards;
-    int64_t row_base;     // first row this shard holds
-    void *block;          // phase 1: this shard's exchange block
-    const void *blocks;   // phase 2: every shard's block, in shard order
-    size_t block_bytes;
-    size_t block_rsum;    // offset of the fp64 row sums inside a block
+    int phase;                        // 1: reduce, local exponents; 2: pack at the global
+                                      // exponents; 3: state pass and apply
+    int cta_begin, cta_end;           // this shard's CTAs of the whole-table grid
+    int64_t row_base;                 // first row this shard holds
+    unsigned char *scales;            // D + 1 exponents: phase 1 out, phases 2 and 3 in (all-reduced by max)
+    unsigned long long *sums;         // D + 1 fixed-point totals: phase 2 out, phase 3 in (all-reduced by sum)
 };
 
 struct DenseArgs {
@@ -166,21 +170,71 @@ struct DenseArgs {
     float *G_stage;            // nullptr, or the HBM copy the reduce pass writes of a host-resident G
     const LmArgs *lm;          // nullptr, or: G is formed by the LM-head kernel instead of read
     const ShardArgs *shard;    // nullptr, or: one phase of a row-sharded step
+    uint64_t wait_ns;          // limit of every bounded wait inside a kernel
 };
 
-// CTAs of the dense step's reduce and apply grids for a V-row table.
-inline int dense_parts(int64_t V) { return (int)(V < kGridCtas ? V : kGridCtas); }
+// CTAs of the dense step's reduce and apply grids for a V x D table: one
+// per kMinCtaElems elements of G (so that a table of up to 8 x 8192
+// elements has at most 8 CTAs and runs as one cluster launch), at most
+// kGridCtas and at most one per row.  A function of (V, D) only, so the
+// per-CTA partial sums -- and the results -- are the same on every run and
+// device.
+constexpr int64_t kMinCtaElems = 8192;
+inline int dense_parts(int64_t V, int64_t D)
+{
+    int64_t n = (V * D + kMinCtaElems - 1) / kMinCtaElems;
+    if (n > kGridCtas)
+        n = kGridCtas;
+    if (n > V)
+        n = V;
+    return (int)(n < 1 ? 1 : n);
+}
+
+// Default limit of a bounded wait inside a kernel (grid barriers, mbarrier
+// waits): 2 s of wall time.
+constexpr uint64_t kDefaultWaitNs = 2000000000ull;
 
 cudaError_t launch_dense_step(const DenseArgs &a);
+
+// beta2 r + (1 - beta2) m is formed in fp32 with each coefficient carried as
+// a float pair hi + lo (hi the coefficient rounded to fp32, lo the rest),
+// computed once on the host.  See ema_pair() in ember_dense.cu.
+struct EmaPair {
+    float bh, bl, ah, al;
+};
+
+// Constants of one step, rounded to fp32 on the host: the EMA coefficients,
+// 1/D, 1/V and the bias-correction factor 1/(1 - beta2^t) (1 without it).
+// GB300 runs fp64 at a small fraction of its fp32 rate, so the kernels keep
+// fp64 out of their latency-bound parts.
+struct StepConsts {
+    EmaPair ema;
+    float inv_D, inv_V, inv_bc;
+};
+inline StepConsts make_consts(double beta2, double one_minus_beta2, int64_t V, int64_t D, double inv_bc)
+{
+    StepConsts k;
+    k.ema.bh = (float)beta2;
+    k.ema.bl = (float)(beta2 - (double)k.ema.bh);
+    k.ema.ah = (float)one_minus_beta2;
+    k.ema.al = (float)(one_minus_beta2 - (double)k.ema.ah);
+    k.inv_D = (float)(1.0 / (double)D);
+    k.inv_V = (float)(1.0 / (double)V);
+    k.inv_bc = (float)inv_bc;
+    return k;
+}
 
 // Column EMA and normaliser; with nrow_ctas > 0 the same launch also runs a
 // row pass: r for all V rows from per-slice sums of g^2, taken from
 // rowpart[slot[i]-1][nslices] for the sparse step (rows with slot 0 saw no
 // gradient) or, with slot == nullptr, from rowpart[nslices][V] for every row.
-cudaError_t launch_state(const float *colpart, int nparts, double *rsum_part, int nrsum, float *c,
-                         double *csum_part, DevScalars *sc, int64_t V, int D, double beta2,
-                         double one_minus_beta2, double inv_bc, cudaStream_t stream, bool pdl,
-                         float *r_rows, int32_t *slot, const float *rowpart, int nslices, int nrow_ctas);
+// Column totals are exact fixed-point sums of the nparts partial rows
+// (ember_device.cuh); the normaliser's sum of r likewise over the nrsum
+// per-CTA sums in rsum_part.
+cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
+                         float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &k,
+                         cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
+                         int nslices, int nrow_ctas);
 
 struct SparseArgs {
     int64_t V, D, N;
@@ -243,4 +297,5 @@ struct ember_handle {
     int64_t ws_max_N;
     cudaEvent_t trace[ember::kMaxTraceEvents];
     int n_trace;
+    uint64_t wait_ns;  // limit of the bounded waits inside kernels (ember_set_wait_limit_ns)
 };

@@ -49,9 +49,10 @@
 // order, whatever the grid; nothing is accumulated across CTAs here.  The
 // state pass sums the per-tile partials in a fixed order.
 //
-// Waits on mbarriers are bounded (kWaitNs of wall time); a wait that gives up
-// sets the sticky timeout flag, stops every role, lets the copies and MMAs
-// already issued finish, frees the tensor memory and returns.
+// Waits on mbarriers are bounded (the handle's wait limit, 2 s by default, of
+// wall time); a wait that gives up sets the sticky timeout flag, stops every
+// role, lets the copies and MMAs already issued finish (those teardown waits
+// keep the fixed 2 s limit), frees the tensor memory and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_runtime.h>
@@ -139,25 +140,28 @@ __device__ __forceinline__ bool mbar_test(uint32_t bar, uint32_t parity)
 }
 
 // Wait for the phase of parity `parity` of `bar` to complete.  Gives up when
-// another role has aborted or after kWaitNs; returns false then.
-__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort)
+// another role has aborted or after limit_ns (the handle's wait limit);
+// returns false then.
+__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort, uint64_t limit_ns)
 {
     if (mbar_test(bar, parity))
         return true;
+    // try_wait may suspend the thread for a while before it reports "not
+    // yet", so the clock and the abort word are checked after every try
     const uint64_t t0 = now_ns();
-    for (uint32_t k = 1;; ++k) {
+    for (;;) {
         if (mbar_test(bar, parity))
             return true;
-        if ((k & 63u) == 0) {
-            if (*abort)
-                return false;
-            if (now_ns() - t0 > kWaitNs)
-                return false;
-        }
+        if (*abort)
+            return false;
+        if (now_ns() - t0 > limit_ns)
+            return false;
     }
 }
 
-// Same, for teardown: no abort check, only the time limit.
+// Same, for teardown: no abort check, only the fixed limit kWaitNs (the
+// copies and MMAs already issued are waited for even when the main-loop
+// limit was made short).
 __device__ bool mbar_wait_final(uint32_t bar, uint32_t parity)
 {
     const uint64_t t0 = now_ns();
@@ -368,7 +372,7 @@ __device__ __forceinline__ void tile_of(int gt, int nblocks, int mpairs, int ban
 __global__ void __launch_bounds__(kLmThreads, 1)
 k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__ CUtensorMap tm_h,
               const __grid_constant__ CUtensorMap tm_g, float *__restrict__ colpart, float *__restrict__ rowpart,
-              unsigned *flags, int V, int D, int T, int band)
+              unsigned *flags, int V, int D, int T, int band, uint64_t wait_ns)
 {
     extern __shared__ unsigned char lm_smem_raw[];
     unsigned char *smem = reinterpret_cast<unsigned char *>(
@@ -438,7 +442,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
             tile_of(gt, nblocks, mpairs, band, rank, mb, nb);
             for (int kb = 0; kb < kblocks; ++kb) {
                 // both CTAs' halves of this stage were read by the pair's MMAs
-                if (!mbar_wait(smem_addr(&tail->empty[stage]), phase ^ 1u, abort)) {
+                if (!mbar_wait(smem_addr(&tail->empty[stage]), phase ^ 1u, abort, wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -482,14 +486,14 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         uint32_t acc_phase = 0;
         bool ok = true;
         for (int gt = gt0; gt < npair_tiles && ok; gt += gstep) {
-            if (!mbar_wait(smem_addr(&tail->tempty[acc]), acc_phase ^ 1u, abort)) {
+            if (!mbar_wait(smem_addr(&tail->tempty[acc]), acc_phase ^ 1u, abort, wait_ns)) {
                 ok = false;
                 break;
             }
             tc_fence_after();
             const uint32_t d_tmem = tmem + (uint32_t)(acc * kAccCols);
             for (int kb = 0; kb < kblocks; ++kb) {
-                if (!mbar_wait(smem_addr(&tail->full[stage]), phase, abort)) {
+                if (!mbar_wait(smem_addr(&tail->full[stage]), phase, abort, wait_ns)) {
                     ok = false;
                     break;
                 }
@@ -535,7 +539,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         for (int gt = gt0; gt < npair_tiles; gt += gstep) {
             int mb, nb;
             tile_of(gt, nblocks, mpairs, band, rank, mb, nb);
-            bool fail = !mbar_wait(smem_addr(&tail->tfull[acc]), acc_phase, abort);
+            bool fail = !mbar_wait(smem_addr(&tail->tfull[acc]), acc_phase, abort, wait_ns);
             if (fail && !*abort)
                 set_timeout(abort, flags);
             fail = fail || *abort;
@@ -697,7 +701,7 @@ cudaError_t launch_lmhead_grad(const LmArgs &a, float *colpart, float *rowpart, 
     cfg.gridDim = dim3(nclusters * 2);
     const int band = kLmBand < lmhead_col_blocks(a.D) ? kLmBand : lmhead_col_blocks(a.D);
     return cudaLaunchKernelEx(&cfg, k_lmhead_grad, tm_dl, tm_h, tm_g, colpart, rowpart, flags, (int)a.V,
-                              (int)a.D, (int)a.T, band);
+                              (int)a.D, (int)a.T, band, a.wait_ns ? a.wait_ns : kDefaultWaitNs);
 }
 
 }  // namespace ember

@@ -7,10 +7,9 @@
 //     fully reserved;
 //   - code paths where a cudaMalloc would synchronise the device in the
 //     middle of a training step.
-// For them this entry point runs the very same three kernels as
-// ember_step_dense, with their scratch (per-CTA column partials, row-sum
-// partials, a few scalars) in a file-scope device array instead of a bound
-// workspace.  It allocates nothing: no cudaMalloc, no cudaFree, no allocating
+// For them this entry point runs the very same kernels as ember_step_dense,
+// with their scratch (per-CTA column partials, row-sum partials, a few
+// scalars) in a file-scope device array instead of a bound workspace.  It allocates nothing: no cudaMalloc, no cudaFree, no allocating
 // library call.
 //
 // The array is kNoAllocScratchBytes (10 MiB) on every GPU that loads the
@@ -19,8 +18,14 @@
 // column panels with per-row partial sums, are refused.
 //
 // In host code the array's name is only a host-side stand-in; the kernels get
-// its device address, looked up once per device with cudaGetSymbolAddress on
-// the first call made with that device current.
+// its device address, looked up with cudaGetSymbolAddress on the first call
+// made with a device current.  The address is cached per device together
+// with the CUDA context it was looked up in: after a cudaDeviceReset (or any
+// teardown and re-creation of the device's context) the module is loaded
+// again, the context differs, and the address is looked up again instead of
+// reusing a stale one.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <math.h>
 #include <mutex>
@@ -36,22 +41,54 @@ constexpr int kMaxDevices = 64;
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocScratchBytes];
 
 std::mutex g_setup_mutex;
-unsigned char *g_scratch_addr[kMaxDevices] = {};
+struct ScratchAddr {
+    CUcontext ctx;
+    unsigned char *ptr;
+};
+ScratchAddr g_scratch[kMaxDevices] = {};
 
-// Device address of the scratch array on the current device (nullptr on error).
+// The driver's cuCtxGetCurrent, reached through the runtime (no link to
+// libcuda needed); nullptr if the driver does not provide it.
+PFN_cuCtxGetCurrent_v4000 ctx_get_current_fn()
+{
+    static PFN_cuCtxGetCurrent_v4000 fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 4000, cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuCtxGetCurrent_v4000>(p);
+    });
+    return fn;
+}
+
+// Device address of the scratch array on the current device and context
+// (nullptr on error).
 unsigned char *scratch_for_current_device()
 {
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices)
         return nullptr;
+    PFN_cuCtxGetCurrent_v4000 get_ctx = ctx_get_current_fn();
+    if (!get_ctx)
+        return nullptr;
     std::lock_guard<std::mutex> lock(g_setup_mutex);
-    if (!g_scratch_addr[dev]) {
+    CUcontext ctx = nullptr;
+    if (get_ctx(&ctx) != CUDA_SUCCESS)
+        return nullptr;
+    if (!ctx || !g_scratch[dev].ptr || g_scratch[dev].ctx != ctx) {
+        // the lookup also makes the device's primary context current if no
+        // runtime call has yet; the context is read again after it
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p)
             return nullptr;
-        g_scratch_addr[dev] = static_cast<unsigned char *>(p);
+        if (get_ctx(&ctx) != CUDA_SUCCESS || !ctx)
+            return nullptr;
+        g_scratch[dev].ctx = ctx;
+        g_scratch[dev].ptr = static_cast<unsigned char *>(p);
     }
-    return g_scratch_addr[dev];
+    return g_scratch[dev].ptr;
 }
 
 bool aligned(const void *p, size_t a) { return ((uintptr_t)p % a) == 0; }
@@ -71,7 +108,8 @@ extern "C" ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const
         return EMBER_ERR_ALIGNMENT;
 
     // The dense kernels use the workspace's scalars, row-sum partials,
-    // column-sum partials of one CTA grid, nothing after that.
+    // column-group sums and the column-sum partials of one CTA grid (at most
+    // kGridCtas rows of D floats), nothing after that.
     const Layout lay = make_layout(h->V, h->D, 0);
     const size_t need = lay.colpart + sizeof(float) * (size_t)kGridCtas * (size_t)h->D;
     if (need > kNoAllocScratchBytes)
@@ -111,6 +149,7 @@ extern "C" ember_status ember_step_dense_noalloc(ember_handle *h, void *W, const
     a.lay = lay;
     a.stream = s;
     a.trace = nullptr;
+    a.wait_ns = h->wait_ns;
     a.map = map;
     return launch_dense_step(a) == cudaSuccess ? EMBER_OK : EMBER_ERR_CUDA;
 }

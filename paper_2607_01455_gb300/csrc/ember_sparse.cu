@@ -846,8 +846,8 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     auto *bounds = reinterpret_cast<int32_t *>(ws + L.sp_bounds);
     auto *S = reinterpret_cast<float *>(ws + L.sp_rows);
     auto *colpart = reinterpret_cast<float *>(ws + L.colpart);
-    auto *rsum_part = reinterpret_cast<double *>(ws + L.rsum_part);
-    auto *csum_part = reinterpret_cast<double *>(ws + L.csum_part);
+    auto *rsum_part = reinterpret_cast<float *>(ws + L.rsum_part);
+    auto *csum_part = reinterpret_cast<float *>(ws + L.csum_part);
     const int D = (int)a.D;
     const int DV = D / VEC;
     const int NS = (DV + kThreads - 1) / kThreads;
@@ -866,8 +866,9 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     // row pass (all V rows) and column pass in one launch
     const int64_t vb = (a.V + (int64_t)kStateThreads * kRowBatch - 1) / ((int64_t)kStateThreads * kRowBatch);
     const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
-    launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, a.beta2, a.one_minus_beta2,
-                 a.inv_bc, a.stream, tr.pdl(), a.r, slot, rowpart, NS, GV);
+    const StepConsts kc = make_consts(a.beta2, a.one_minus_beta2, a.V, a.D, a.inv_bc);
+    launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, kc, a.stream, tr.pdl(), a.r, slot, rowpart,
+                 NS, GV);
     tr.mark();
     // one launch per column panel (one unless D is wider than a CTA's row)
     const int np = a.map.npanels, pw = a.map.pw;

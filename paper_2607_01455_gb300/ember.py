@@ -39,8 +39,8 @@ EXPORTS = (
     "ember_abi_version", "ember_set_trace_events", "ember_sparse_unique",
     "ember_step_dense_noalloc", "ember_step_dense_from_host",
     "ember_lmhead_grad", "ember_step_lmhead",
-    "ember_shard_rows", "ember_shard_exchange_bytes", "ember_shard_reduce", "ember_shard_update",
-    "ember_column_panels",
+    "ember_shard_rows", "ember_shard_scale_bytes", "ember_shard_exchange_bytes", "ember_shard_reduce",
+    "ember_shard_pack", "ember_shard_update", "ember_column_panels", "ember_set_wait_limit_ns",
 )
 
 
@@ -90,10 +90,13 @@ def lib():
             "ember_lmhead_grad": (st, [vp, vp, vp, i64, vp, vp]),
             "ember_step_lmhead": (st, [vp, vp, vp, vp, i64, vp, vp, flt, i64, vp]),
             "ember_shard_rows": (i64, [vp, ip, ip, ctypes.POINTER(i64)]),
-            "ember_shard_exchange_bytes": (sz, [vp, ip]),
+            "ember_shard_scale_bytes": (sz, [vp]),
+            "ember_shard_exchange_bytes": (sz, [vp]),
             "ember_shard_reduce": (st, [vp, ip, ip, vp, vp, vp, vp]),
-            "ember_shard_update": (st, [vp, ip, ip, vp, vp, vp, vp, flt, i64, vp]),
+            "ember_shard_pack": (st, [vp, ip, ip, vp, vp, vp]),
+            "ember_shard_update": (st, [vp, ip, ip, vp, vp, vp, vp, vp, flt, i64, vp]),
             "ember_column_panels": (ip, [vp, ip]),
+            "ember_set_wait_limit_ns": (st, [vp, ctypes.c_uint64]),
         }
         for name, (res, args) in sig.items():
             fn = getattr(L, name)
@@ -208,18 +211,34 @@ def ember_shard_rows(h, shard, nshards):
     return row0.value, n
 
 
-def ember_shard_exchange_bytes(h, nshards):
-    return lib().ember_shard_exchange_bytes(h, nshards)
+def ember_shard_scale_bytes(h):
+    """Bytes of a shard's exponent block (one uint8 per column, one for the r sums)."""
+    return lib().ember_shard_scale_bytes(h)
 
 
-def ember_shard_reduce(h, shard, nshards, G_shard, state, block, stream=None):
-    _check(lib().ember_shard_reduce(h, shard, nshards, _addr(G_shard), _addr(state), _addr(block),
+def ember_shard_exchange_bytes(h):
+    """Bytes of a shard's fixed-point block (one uint64 per column, one for the r sums)."""
+    return lib().ember_shard_exchange_bytes(h)
+
+
+def ember_shard_reduce(h, shard, nshards, G_shard, state, scales, stream=None):
+    _check(lib().ember_shard_reduce(h, shard, nshards, _addr(G_shard), _addr(state), _addr(scales),
                                     _stream(stream)), "ember_shard_reduce")
 
 
-def ember_shard_update(h, shard, nshards, W_shard, G_shard, state, blocks, lr, t, stream=None):
+def ember_shard_pack(h, shard, nshards, scales, sums, stream=None):
+    _check(lib().ember_shard_pack(h, shard, nshards, _addr(scales), _addr(sums), _stream(stream)),
+           "ember_shard_pack")
+
+
+def ember_shard_update(h, shard, nshards, W_shard, G_shard, state, scales, sums, lr, t, stream=None):
     _check(lib().ember_shard_update(h, shard, nshards, _addr(W_shard), _addr(G_shard), _addr(state),
-                                    _addr(blocks), lr, t, _stream(stream)), "ember_shard_update")
+                                    _addr(scales), _addr(sums), lr, t, _stream(stream)), "ember_shard_update")
+
+
+def ember_set_wait_limit_ns(h, ns):
+    """Limit of the bounded waits inside this handle's kernels (0: the default, 2 s)."""
+    _check(lib().ember_set_wait_limit_ns(h, int(ns)), "ember_set_wait_limit_ns")
 
 
 def ember_step_sparse(h, W, ids, idtype, N, rows, state, lr, t, stream=None):
@@ -299,14 +318,24 @@ class Ember:
     def shard_rows(self, shard, nshards):
         return ember_shard_rows(self.handle, shard, nshards)
 
-    def shard_exchange_bytes(self, nshards):
-        return ember_shard_exchange_bytes(self.handle, nshards)
+    def shard_scale_bytes(self):
+        return ember_shard_scale_bytes(self.handle)
 
-    def shard_reduce(self, shard, nshards, G_shard, block, stream=None):
-        ember_shard_reduce(self.handle, shard, nshards, G_shard, self.state, block, stream)
+    def shard_exchange_bytes(self):
+        return ember_shard_exchange_bytes(self.handle)
 
-    def shard_update(self, shard, nshards, W_shard, G_shard, blocks, lr, t, stream=None):
-        ember_shard_update(self.handle, shard, nshards, W_shard, G_shard, self.state, blocks, lr, t, stream)
+    def shard_reduce(self, shard, nshards, G_shard, scales, stream=None):
+        ember_shard_reduce(self.handle, shard, nshards, G_shard, self.state, scales, stream)
+
+    def shard_pack(self, shard, nshards, scales, sums, stream=None):
+        ember_shard_pack(self.handle, shard, nshards, scales, sums, stream)
+
+    def shard_update(self, shard, nshards, W_shard, G_shard, scales, sums, lr, t, stream=None):
+        ember_shard_update(self.handle, shard, nshards, W_shard, G_shard, self.state, scales, sums, lr, t,
+                           stream)
+
+    def set_wait_limit_ns(self, ns):
+        ember_set_wait_limit_ns(self.handle, ns)
 
     def step_sparse(self, W, ids, rows, lr, t, stream=None):
         import torch

@@ -31,7 +31,7 @@ def test_library_exports_every_declared_function():
     lib = ctypes.CDLL(E.LIB_PATH)
     for name in declared:
         assert hasattr(lib, name), name
-    assert E.ember_abi_version() == 1
+    assert E.ember_abi_version() == 2
 
 
 def test_status_strings():

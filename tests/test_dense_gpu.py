@@ -250,3 +250,30 @@ def test_step_from_host_refuses_unregistered_memory(cuda_device):
     with pytest.raises(EmberError) as ex:
         emb.step_dense_from_host(W, pageable.ctypes.data, stage, 1e-3, 1)
     assert ex.value.status == 1  # EMBER_ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("V,D,wdtype", [(1024, 64, "f32"), (256, 256, "bf16"), (100, 300, "f32"), (1, 4, "bf16"),
+                                         (305, 132, "bf16"), (7, 12, "f32"), (2048, 32, "bf16"),
+                                         (3001, 1024, "bf16"), (40, 8192, "bf16")])
+def test_one_launch_and_three_launch_forms_agree_bitwise(cuda_device, V, D, wdtype):
+    """A small table runs as one cluster launch (G and W kept in shared
+    memory, the column statistics exchanged through distributed shared
+    memory) and, while trace events are set, as three launches (reduce,
+    state, apply).  Both run the same arithmetic on the same CTA row ranges,
+    with the column totals summed exactly, so they give the same bits (the
+    last two shapes take three launches either way)."""
+    a, b = make(V, D, wdtype), make(V, D, wdtype)
+    Wa = rand_w(V, D, wdtype, cuda_device, seed=5)
+    Wb = Wa.clone()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    b.trace(ev)
+    for t in range(1, 5):
+        G = rand_grad(V, D, t, cuda_device, seed=D)
+        a.step_dense(Wa, G, 1e-3, t)
+        b.step_dense(Wb, G, 1e-3, t)
+    torch.cuda.synchronize()
+    b.trace([])
+    view = torch.int16 if wdtype == "bf16" else torch.int32
+    assert torch.equal(Wa.view(view), Wb.view(view))
+    assert torch.equal(a.state.view(torch.int32), b.state.view(torch.int32))
+    assert a.device_status() == 0 and b.device_status() == 0

@@ -237,3 +237,40 @@ def test_step_lmhead_graph_capture_matches_eager(cuda_device):
     assert torch.equal(G1.view(torch.int32), G2.view(torch.int32))
     assert torch.equal(W1.view(torch.int16), W2.view(torch.int16))
     assert torch.equal(e1.state.view(torch.int32), e2.state.view(torch.int32))
+
+
+def test_bounded_wait_gives_up_and_the_next_step_recovers(cuda_device):
+    """The LM-head kernel's main-loop mbarrier waits, made 1 ns long, give up
+    for real: the kernel stops every role, lets the copies and MMAs it has
+    issued complete (its teardown waits keep their 2 s limit), frees its
+    tensor memory and returns, and the sticky flag reads EMBER_ERR_TIMEOUT.
+    The context stays usable: back at the default limit, the fused step on
+    the same handle passes the oracle gate."""
+    from paper_2607_01455_gb300.ember import EMBER_ERR_TIMEOUT
+    V, D, T = 2048, 1024, 4096  # 64 pipeline stages per tile: many waits
+    emb = make(V, D, "f32")
+    dl, h = synth.lmhead_inputs(V, D, T, seed=9, t=1, device=cuda_device)
+    G = torch.zeros(V, D, device=cuda_device)
+    emb.set_wait_limit_ns(1)
+    emb.lmhead_grad(dl, h, G)
+    assert emb.device_status() == EMBER_ERR_TIMEOUT
+    assert emb.device_status() == 0  # read and cleared
+    emb.set_wait_limit_ns(0)
+    gw = torch.Generator(device=cuda_device).manual_seed(4)
+    W = torch.randn(V, D, generator=gw, device=cuda_device) * 0.02
+    for t in (1, 2):
+        dl, h = synth.lmhead_inputs(V, D, T, seed=9, t=t, device=cuda_device)
+        W0 = w_to_host(W)
+        st0 = emb.state.cpu().numpy().copy()
+        emb.step_lmhead(W, dl, h, G, 1e-3, t)
+        torch.cuda.synchronize()
+        assert emb.device_status() == 0
+        if t == 1:
+            check_gemm(G, dl, h, rows=np.arange(0, V, 7))
+        r, c = st0[:V].copy(), st0[V:].copy()
+        Wo = W0.copy()
+        oracle.step_dense(Wo, G.cpu().numpy(), r, c, float(np.float32(1e-3)), t)
+        st = emb.state.cpu().numpy()
+        check_state(st[:V], r, "r")
+        check_state(st[V:], c, "c")
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0)

@@ -1,11 +1,12 @@
 """Host side of the row-sharded dense step, on the CPU (no kernel runs).
 
-The shard plan (which rows each shard holds, how big its exchange block
-is) is host logic of the library: it must tile the table exactly at the
-whole-table step's CTA row boundaries, give every shard the same block
-size (what an all-gather needs), and reject bad arguments before any CUDA
-call.  The last test runs the plan on world_size 3 gloo ranks and
-all-gathers it, as ranks of a sharded job would.
+The shard plan (which rows each shard holds, how big its exchange blocks
+are) is host logic of the library: it must tile the table exactly at the
+whole-table step's CTA row boundaries, give every shard blocks of the same
+size (what an all-reduce needs: D + 1 exponent bytes and D + 1 fixed-point
+words, kilobytes rather than the per-CTA partial rows), and reject bad
+arguments before any CUDA call.  The last test runs the plan on world_size
+3 gloo ranks and all-gathers it, as ranks of a sharded job would.
 """
 import os
 import socket
@@ -22,28 +23,42 @@ def built():
     build_library()
 
 
-def cta_rows(V):
-    """Row boundaries of the whole-table step's CTAs (304 per GPU at most)."""
-    nparts = min(V, 304)
+def cta_rows(V, D):
+    """Row boundaries of the whole-table step's CTAs: one per 8192 elements
+    of G, at most 304 (two per SM of the GB300) and at most one per row."""
+    nparts = max(1, min(V, 304, -(-V * D // 8192)))
     return [b * V // nparts for b in range(nparts + 1)]
 
 
-@pytest.mark.parametrize("V", [1, 7, 303, 304, 305, 1000, 128256])
+@pytest.mark.parametrize("V,D", [(1, 16), (7, 16), (303, 16), (304, 2048), (305, 4096), (1000, 16),
+                                 (1000, 200), (128256, 16), (128256, 8192)])
 @pytest.mark.parametrize("n", [1, 2, 3, 4, 8, 300, 305])
-def test_shards_tile_the_table_at_cta_boundaries(V, n):
-    h = E.ember_create(V, 16)
+def test_shards_tile_the_table_at_cta_boundaries(V, D, n):
+    h = E.ember_create(V, D)
     try:
-        bounds = set(cta_rows(V))
+        bounds = set(cta_rows(V, D))
         nxt = 0
-        sizes = set()
         for k in range(n):
             row0, rows = E.ember_shard_rows(h, k, n)
             assert row0 == nxt and rows >= 0
             assert row0 in bounds and row0 + rows in bounds
             nxt = row0 + rows
-            sizes.add(E.ember_shard_exchange_bytes(h, n))
         assert nxt == V
-        assert len(sizes) == 1 and sizes.pop() % 256 == 0
+        # the two blocks every shard all-reduces: one byte and one 64-bit word
+        # per column, and one of each for the sums of r
+        assert E.ember_shard_scale_bytes(h) == D + 1
+        assert E.ember_shard_exchange_bytes(h) == 8 * (D + 1)
+    finally:
+        E.ember_destroy(h)
+
+
+def test_exchange_is_kilobytes_at_the_lm_head_width():
+    """Section 2.3 asks for a kilobyte-scale exchange: at D = 8192 the
+    fixed-point block is 64 KiB and the exponent block 8 KiB."""
+    h = E.ember_create(128256, 8192)
+    try:
+        assert E.ember_shard_exchange_bytes(h) == 65544
+        assert E.ember_shard_scale_bytes(h) == 8193
     finally:
         E.ember_destroy(h)
 
@@ -59,16 +74,27 @@ def test_shard_rejects_on_host():
         assert lib.ember_shard_rows(h, -1, 2, ctypes.byref(r0)) == -1
         assert lib.ember_shard_rows(h, 0, 0, ctypes.byref(r0)) == -1
         assert lib.ember_shard_rows(None, 0, 1, ctypes.byref(r0)) == -1
-        assert lib.ember_shard_exchange_bytes(h, 0) == 0
-        assert lib.ember_shard_reduce(h, 0, 2, fake, fake, fake, None) == E.EMBER_ERR_WORKSPACE
-        assert lib.ember_shard_reduce(h, 3, 2, fake, fake, fake, None) == E.EMBER_ERR_INVALID_ARG
-        assert lib.ember_shard_reduce(h, 0, 2, fake + 4, fake, fake, None) == E.EMBER_ERR_ALIGNMENT
-        assert lib.ember_shard_reduce(h, 0, 2, fake, fake, fake + 64, None) == E.EMBER_ERR_ALIGNMENT
-        assert lib.ember_shard_reduce(h, 0, 2, None, fake, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert lib.ember_shard_exchange_bytes(None) == 0
+        assert lib.ember_shard_scale_bytes(None) == 0
+        red = lib.ember_shard_reduce
+        assert red(h, 0, 2, fake, fake, fake, None) == E.EMBER_ERR_WORKSPACE
+        assert red(h, 3, 2, fake, fake, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert red(h, 0, 2, fake + 4, fake, fake, None) == E.EMBER_ERR_ALIGNMENT
+        assert red(h, 0, 2, fake, fake + 2, fake, None) == E.EMBER_ERR_ALIGNMENT
+        assert red(h, 0, 2, None, fake, fake, None) == E.EMBER_ERR_WORKSPACE  # checked after the plan
+        assert red(h, 0, 2, fake, fake, None, None) == E.EMBER_ERR_INVALID_ARG
+        pk = lib.ember_shard_pack
+        assert pk(h, 0, 2, fake, fake, None) == E.EMBER_ERR_WORKSPACE
+        assert pk(h, 0, 2, None, fake, None) == E.EMBER_ERR_INVALID_ARG
+        assert pk(h, 0, 2, fake, None, None) == E.EMBER_ERR_INVALID_ARG
+        assert pk(h, 0, 2, fake, fake + 4, None) == E.EMBER_ERR_ALIGNMENT
+        assert pk(h, 2, 2, fake, fake, None) == E.EMBER_ERR_INVALID_ARG
         up = lib.ember_shard_update
-        assert up(h, 0, 2, fake, fake, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
-        assert up(h, 0, 2, None, fake, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
-        assert up(h, 0, 2, fake, fake, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
+        assert up(h, 0, 2, fake, fake, fake, fake, fake, 1e-3, 0, None) == E.EMBER_ERR_INVALID_ARG
+        assert up(h, 0, 2, fake, fake, fake, fake, fake, float("nan"), 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert up(h, 0, 2, fake, fake, fake, None, fake, 1e-3, 1, None) == E.EMBER_ERR_INVALID_ARG
+        assert up(h, 0, 2, fake, fake, fake, fake, fake + 4, 1e-3, 1, None) == E.EMBER_ERR_ALIGNMENT
+        assert up(h, 0, 2, fake, fake, fake, fake, fake, 1e-3, 1, None) == E.EMBER_ERR_WORKSPACE
     finally:
         E.ember_destroy(h)
     hp = E.ember_hparams_default()
@@ -93,7 +119,7 @@ def _rank(rank, world, port, V, D, out):
     dist.init_process_group("gloo", rank=rank, world_size=world)
     h = E.ember_create(V, D)
     row0, rows = E.ember_shard_rows(h, rank, world)
-    nbytes = E.ember_shard_exchange_bytes(h, world)
+    nbytes = E.ember_shard_exchange_bytes(h)
     E.ember_destroy(h)
     mine = torch.tensor([row0, rows, nbytes], dtype=torch.int64)
     parts = [torch.zeros(3, dtype=torch.int64) for _ in range(world)]

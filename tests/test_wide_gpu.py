@@ -195,7 +195,7 @@ def test_wide_step_lmhead_gated(cuda_device, V, D, T):
 def test_wide_tables_are_refused_by_shards_and_noalloc(cuda_device):
     V, D = 64, 16384
     emb = make(V, D, "bf16")
-    blk = torch.zeros(emb.shard_exchange_bytes(2), dtype=torch.uint8, device=cuda_device)
+    blk = torch.zeros(emb.shard_scale_bytes(), dtype=torch.uint8, device=cuda_device)
     with pytest.raises(EmberError) as ex:
         emb.shard_reduce(0, 2, torch.zeros(V // 2, D, device=cuda_device), blk)
     assert ex.value.status == E.EMBER_ERR_UNSUPPORTED
