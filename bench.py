@@ -7,13 +7,19 @@ bf16 weights, fp32 gradient and state.  Inputs are resident in HBM when the
 timed region starts; L2 is flushed (a 512 MiB write) between timed steps,
 outside the per-step CUDA events.  `value` is algorithmic bytes per step over
 the mean step time, summed over ranks (independent replicas: the step has no
-cross-GPU exchange on one table held whole by each GPU).
+cross-GPU exchange on one table held whole by each GPU).  The same line
+carries one sub-object per workload of the method (`configs`: the 1024 x 64
+fp32 table, the 32000 x 4096 and 151936 x 896 bf16 tables, the sparse
+262144 x 2048 step with 32768 ids, and the LM head), each with its step
+time, its GB/s and the roofline of its dominant kernel, the fused LM-head
+step, the row-only variant and the CPU oracle on one core and on all cores.
 
   python bench.py [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
 
---impl reference times the CPU oracle (plain C, one core) on a bounded row
-sample of the same workload: the paper ships no implementation to compare
-with, so that is the reference arm.
+--impl reference times the CPU oracle (plain C; its OpenMP build on all host
+cores, which gives the same bits) on a bounded row sample of the same
+workload: the paper ships no implementation to compare with, so that is the
+reference arm.
 """
 import argparse
 import json
@@ -32,16 +38,14 @@ NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
 
-# dram__bytes_read.sum + dram__bytes_write.sum per launch of the apply kernel,
-# by workload (V=128256, D=8192, bf16 W: the default), from the one-pass ncu
-# capture summarised in profiles/dense_lmhead_v128256_d8192_bf16_launches.md.
-# Set to None whenever k_apply_dense changes until it is captured again.
-APPLY_TRAFFIC_BYTES = {"dense_lmhead_v128256_d8192_bf16": 8374828715}
-# The same for k_lmhead_grad on the LM-head gradient workload (V=128256,
-# D=8192, T=4096), from profiles/lmhead_grad_v128256_d8192_t4096_bf16_launches.md.
-# Set to None whenever k_lmhead_grad changes until it is captured again.
-LMHEAD_TRAFFIC_BYTES = {"lmhead_grad_v128256_d8192_t4096_bf16": 11450829184}
-
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of a
+# dominant kernel, from an ncu capture of the kernel as it is now, with where
+# it came from.  A kernel that changes gets None here until it is captured
+# again.
+TRAFFIC = {
+    ("k_apply_dense", "dense_lmhead_v128256_d8192_bf16"): None,
+    ("k_lmhead_grad", "lmhead_grad_v128256_d8192_t4096_bf16"): None,
+}
 
 def wbytes(wl):
     return 2 if wl.wdtype == "bf16" else 4
@@ -82,6 +86,114 @@ def traced_steps(steps):
         raise SystemExit("--steps must be at least 2")
     t = [k for k in range(steps) if k % TRACE_EVERY == TRACE_EVERY - 1]
     return t or [steps - 1]
+
+
+def traffic_of(kernel, name):
+    """{"traffic": bytes or None, "traffic_source": where they came from}."""
+    t = TRAFFIC.get((kernel, name))
+    if t is None:
+        return {"traffic": None, "traffic_source": "not captured for this kernel version"}
+    return {"traffic": t[0], "traffic_source": t[1]}
+
+
+def hbm_roofline(kernel, bytes_per_launch, ms_per_launch, wl_name):
+    peak, peak_kind = measured_hbm_peak()
+    ach = bytes_per_launch / (ms_per_launch * 1e-3) / 1e9
+    return {"bound": "hbm", "kernel": kernel, "achieved": ach, "peak": peak, "unit": "GB/s",
+            "frac": ach / peak, "peak_kind": peak_kind, "algorithmic_bytes_per_launch": bytes_per_launch,
+            **traffic_of(kernel, wl_name)}
+
+
+def run_dense(wl, dev, steps, warmup, flush, seed=0, clocks_for=None):
+    """Times ember_step_dense on one workload (L2 flushed between steps).
+    Untraced steps time the whole step; for a table that runs as three
+    launches, every TRACE_EVERY-th step records events at the kernel
+    boundaries for the per-kernel times (a small table runs as one cluster
+    launch, whose time is the step's)."""
+    import torch
+    from paper_2607_01455_gb300 import synth
+    from paper_2607_01455_gb300.ember import Ember
+    W = synth.init_weights(wl, seed, dev)
+    G = synth.dense_grad(wl, seed, 1, dev)
+    emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
+    vec = wl.D % 4 == 0
+    launches = emb.dense_step_launches(vec)
+    npan = emb.column_panels(vec)
+    three = launches == 2 * npan + 1
+    t = 0
+    warm_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    for i in range(warmup):
+        t += 1
+        flush.zero_()
+        emb.trace(warm_ev if (three and i % 2) else [])
+        emb.step_dense(W, G, wl.lr, t)
+    torch.cuda.synchronize()
+    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    traced = traced_steps(steps) if three else []
+    kern_ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(4)] for k in traced}
+    stream = torch.cuda.current_stream(dev)
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    sampler = clocks_for if clocks_for is not None else _NullClocks()
+    with sampler:
+        for k in range(steps):
+            t += 1
+            flush.zero_()
+            emb.trace(kern_ev.get(k, []))
+            step_ev[k][0].record(stream)
+            emb.step_dense(W, G, wl.lr, t)
+            step_ev[k][1].record(stream)
+        torch.cuda.synchronize()
+    wall = time.perf_counter() - wall0
+    emb.trace([])
+    if emb.device_status() != 0:
+        raise SystemExit(f"device status after the {wl.name} steps")
+    plain = [k for k in range(steps) if k not in kern_ev]
+    ms = sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain)
+    B = step_bytes(wl)
+    peak, _ = measured_hbm_peak()
+    out = {"workload": wl.name, "V": wl.V, "D": wl.D, "w_dtype": wl.wdtype, "steps": steps,
+           "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s", "algorithmic_bytes": B,
+           "frac_of_measured_hbm": B / (ms * 1e-3) / 1e9 / peak,
+           "frac_of_nominal_8TBs": B / (ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
+           "params_per_s": wl.V * wl.D / (ms * 1e-3), "launches_per_step": launches,
+           "gpu_launches": launches * steps, "wall_s_timed_region": wall}
+    if three:
+        kb = kernel_bytes(wl)
+        per = {"reduce": [], "state": [], "apply": [], "traced_step": []}
+        for ev in kern_ev.values():
+            per["reduce"].append(ev[0].elapsed_time(ev[1]))
+            per["state"].append(ev[1].elapsed_time(ev[2]))
+            per["apply"].append(ev[2].elapsed_time(ev[3]))
+            per["traced_step"].append(ev[0].elapsed_time(ev[3]))
+        mean = {k: sum(v) / len(v) for k, v in per.items()}
+        out["kernels"] = {k: {"ms": mean[k], "gbs": kb[k] / (mean[k] * 1e-3) / 1e9}
+                          for k in ("reduce", "state", "apply")}
+        out["ms_per_step_traced"] = mean["traced_step"]
+        # the apply pass is the dominant kernel (2/3 of the bytes); with
+        # column panels its launches are per panel and the figures per pass
+        out["roofline"] = hbm_roofline("k_apply_dense", kb["apply"], mean["apply"], wl.name)
+        if npan > 1:
+            out["roofline"]["launches_per_pass"] = npan
+        out["timing"] = (f"step time: CUDA events around each untraced step; kernel times: every "
+                         f"{TRACE_EVERY}th step records events at kernel boundaries")
+    else:
+        # one cluster launch: G read from HBM once, W read and written, the
+        # state read and written once
+        w = wbytes(wl)
+        kbytes = (4 + 2 * w) * wl.V * wl.D + 8 * (wl.V + wl.D)
+        out["kernels"] = {"cluster": {"ms": ms, "gbs": kbytes / (ms * 1e-3) / 1e9}}
+        out["roofline"] = hbm_roofline("k_dense_cluster", kbytes, ms, wl.name)
+        out["timing"] = "CUDA events around each step (one kernel launch per step)"
+    return out
+
+
+class _NullClocks:
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        return False
 
 
 def run_sparse(wl, dev, steps, warmup, flush, seed=0):
@@ -140,7 +252,12 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
     torch.cuda.synchronize()
     ms_graph = sum(a.elapsed_time(b) for a, b in gev) / steps
     B = sparse_bytes(wl, U)
+    kb = sparse_kernel_bytes(wl, U)
+    peak, _ = measured_hbm_peak()
     return {"workload": wl.name, "ms_per_step_graph": ms_graph, "V": wl.V, "D": wl.D, "N": wl.N, "unique_ids": U,
+            "roofline": hbm_roofline("k_sp_segsum", kb["segsum"], per["segsum"], wl.name),
+            "frac_of_measured_hbm": B / (ms * 1e-3) / 1e9 / peak,
+            "frac_of_nominal_8TBs": B / (ms * 1e-3) / 1e9 / NOMINAL_HBM_GBS,
             "ms_per_step": ms, "value": B / (ms * 1e-3) / 1e9, "unit": "GB/s",
             "algorithmic_bytes": B, "touched_params_per_s": U * wl.D / (ms * 1e-3),
             "occurrence_params_per_s": wl.N * wl.D / (ms * 1e-3),
@@ -268,7 +385,8 @@ def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
             "roofline": {"bound": "tensor", "kernel": "k_lmhead_grad", "achieved": tf, "peak": peaks["burst"],
                          "unit": "TFLOP/s", "frac": tf / peaks["burst"],
                          "frac_of_sustained": tf / peaks["sustained"], "peak_kind": peak_kind,
-                         "flops_per_launch": flops, "traffic": LMHEAD_TRAFFIC_BYTES.get(wl.name),
+                         "flops_per_launch": flops,
+                         **traffic_of("k_lmhead_grad", wl.name),
                          "algorithmic_dram_bytes_per_launch": 2 * T * (V + D) + 4 * V * D},
             "unfused": {"ms_per_step": ms_unfused, "cublas_gemm_ms": ms_cublas, "cublas_tflops": tf_cublas,
                         "cublas_output": cublas_out,
@@ -288,7 +406,7 @@ def measured_hbm_peak():
 
 
 class ClockSampler:
-    """nvidia-smi clocks and throttle reasons, sampled every 100 ms."""
+    """nvidia-smi clocks and throttle reasons, sampled every 20 ms."""
     FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
@@ -307,7 +425,7 @@ class ClockSampler:
             self.out = open(self.path, "w")
             self.proc = subprocess.Popen(
                 ["nvidia-smi", "-i", str(self.gpu_index), f"--query-gpu={self.FIELDS}",
-                 "--format=csv,noheader,nounits", "-lms", "100"],
+                 "--format=csv,noheader,nounits", "-lms", "20"],
                 stdout=self.out, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
@@ -359,20 +477,31 @@ class OracleSample:
         self.lr, self.t, self.rows = wl.lr, 0, rows
         self.bytes = step_bytes(sub)
 
-    def step(self):
-        """One oracle step; returns its seconds."""
+    def step(self, all_cores=False):
+        """One oracle step; returns its seconds.  all_cores: the OpenMP build
+        of the same source on every host core (the same bits)."""
         import oracle
         self.t += 1
         t0 = time.perf_counter()
-        oracle.step_dense(self.W, self.G, self.r, self.c, self.lr, self.t)
+        oracle.step_dense(self.W, self.G, self.r, self.c, self.lr, self.t, all_cores=all_cores)
         return time.perf_counter() - t0
 
 
-def sample_rows_for(wl, seconds):
+def host_cores():
+    """Threads the all-cores oracle uses: every core this process may run on."""
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+def sample_rows_for(wl, seconds, all_cores=False):
     """Rows of a sample whose oracle step takes about `seconds`."""
-    probe = 64
-    dt = OracleSample(wl, probe).step()
-    return int(max(16, min(wl.V, probe * seconds / max(dt, 1e-6))))
+    probe = 64 if not all_cores else 1024
+    smp = OracleSample(wl, min(probe, wl.V))
+    smp.step(all_cores)  # the first call loads the library and starts the threads
+    dt = smp.step(all_cores)
+    return int(max(16, min(wl.V, smp.rows * seconds / max(dt, 1e-6))))
 
 
 def dist_setup():
@@ -402,26 +531,29 @@ def allreduce_max(world, x):
 
 
 def run_reference(args, world, rank):
+    import oracle
     from paper_2607_01455_gb300 import synth
     wl = synth.WORKLOADS[args.workload]
     if rank != 0:
         return 0
+    cores = oracle.threads(host_cores())
     budget = 90.0  # seconds of oracle work for the whole warm-up + timed run
-    rows = sample_rows_for(wl, budget / (args.steps + args.warmup))
+    rows = sample_rows_for(wl, budget / (args.steps + args.warmup), all_cores=True)
     smp = OracleSample(wl, rows)
     for _ in range(args.warmup):
-        smp.step()
-    times = [smp.step() for _ in range(args.steps)]
+        smp.step(all_cores=True)
+    times = [smp.step(all_cores=True) for _ in range(args.steps)]
     sec = sum(times) / len(times)
     gbs = smp.bytes / sec / 1e9
-    sample = f"oracle dense step on the first {rows} of {wl.V} rows (D={wl.D}, {wl.wdtype} W), one thread"
+    sample = (f"oracle dense step on the first {rows} of {wl.V} rows (D={wl.D}, {wl.wdtype} W), "
+              f"OpenMP build on {cores} threads")
     line = {
         "impl": "reference", "metric": METRIC, "value": gbs, "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": sec * 1e3,
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic", "config": {"workload": wl.name, "V": wl.V, "D": wl.D,
                                         "w_dtype": wl.wdtype, "sample_rows": rows},
-        "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": gbs, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": gbs, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -443,9 +575,6 @@ def run_sparse_line(args, wl, world, rank, dev):
         sp = run_sparse(wl, dev, args.steps, args.warmup, flush, seed=rank)
         barrier(world)
     ms = allreduce_max(world, sp["ms_per_step"])
-    peak, peak_kind = measured_hbm_peak()
-    kb = sparse_kernel_bytes(wl, sp["unique_ids"])
-    ach = kb["segsum"] / (sp["kernels_ms"]["segsum"] * 1e-3) / 1e9
     line = {
         "metric": METRIC, "value": world * sp["algorithmic_bytes"] / (ms * 1e-3) / 1e9, "unit": "GB/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms,
@@ -454,9 +583,7 @@ def run_sparse_line(args, wl, world, rank, dev):
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "w_dtype": wl.wdtype,
                    "ids": "int64", "l2": "flushed between steps (512 MiB write, outside the events)",
                    "parallelism": f"replicas x{world}"},
-        "roofline": {"bound": "hbm", "kernel": "k_sp_segsum", "achieved": ach, "peak": peak,
-                     "unit": "GB/s", "frac": ach / peak, "peak_kind": peak_kind, "traffic": None,
-                     "algorithmic_bytes_per_launch": kb["segsum"]},
+        "roofline": sp["roofline"],
         "cpu_baseline": None, "e2e": None, "gpu_launches": sp["gpu_launches"],
         "clocks": clocks.summary(), "sparse": sp,
     }
@@ -492,6 +619,14 @@ def run_lmhead_line(args, wl, world, rank, dev):
     return 0
 
 
+CONFIGS = (  # the method's workloads, reported in every default run
+    ("c1", "dense_v1024_d64_f32", 400),
+    ("c2", "dense_v32000_d4096_bf16", 100),
+    ("c3", "dense_tied_v151936_d896_bf16", 100),
+    ("c4", "sparse_v262144_d2048_bf16_n32768", 100),
+)
+
+
 def run_ours(args, world, rank, local):
     import torch
     from paper_2607_01455_gb300 import synth
@@ -506,150 +641,119 @@ def run_ours(args, world, rank, local):
     if wl.kind == "sparse":
         return run_sparse_line(args, wl, world, rank, dev)
 
-    W = synth.init_weights(wl, rank, dev)
-    G = synth.dense_grad(wl, rank, 1, dev)
     flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
-    emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
-    # column panels of this table (one reduce and one apply launch each)
-    npan = emb.column_panels(wl.D % 4 == 0)
-
-    def one_step(t, ev):
-        emb.trace(ev)
-        emb.step_dense(W, G, wl.lr, t)
-
-    warm_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
-    # warm-up alternates traced and untraced steps
-    t = 0
-    for i in range(args.warmup):
-        t += 1
-        flush.zero_()
-        one_step(t, warm_ev if i % 2 else [])
-    torch.cuda.synchronize()
-
-    # untraced steps time the whole step (kernels overlap their launches);
-    # every TRACE_EVERY-th step records kernel boundaries instead
-    step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-               for _ in range(args.steps)]
-    traced = traced_steps(args.steps)
-    events = {k: [torch.cuda.Event(enable_timing=True) for _ in range(4)] for k in traced}
-    barrier(world)
-    torch.cuda.synchronize()
-    wall0 = time.perf_counter()
-    with ClockSampler(local) as clocks:
-        for k in range(args.steps):
-            t += 1
-            flush.zero_()
-            emb.trace(events.get(k, []))
-            step_ev[k][0].record(stream)
-            emb.step_dense(W, G, wl.lr, t)
-            step_ev[k][1].record(stream)
-        torch.cuda.synchronize()
-        barrier(world)
-    wall = time.perf_counter() - wall0
-    emb.trace([])
-    status = emb.device_status()
-    if status != 0:
-        raise SystemExit(f"device status {status} after the timed steps")
-
-    per = {"reduce": [], "state": [], "apply": [], "traced_step": []}
-    for ev in events.values():
-        per["reduce"].append(ev[0].elapsed_time(ev[1]))
-        per["state"].append(ev[1].elapsed_time(ev[2]))
-        per["apply"].append(ev[2].elapsed_time(ev[3]))
-        per["traced_step"].append(ev[0].elapsed_time(ev[3]))
-    mean = {k: sum(v) / len(v) for k, v in per.items()}
-    plain = [k for k in range(args.steps) if k not in events]
-    ms = allreduce_max(world, sum(step_ev[k][0].elapsed_time(step_ev[k][1]) for k in plain) / len(plain))
-
-    B = step_bytes(wl)
-    value = world * B / (ms * 1e-3) / 1e9
     peak, peak_kind = measured_hbm_peak()
-    kb = kernel_bytes(wl)
-    kern = {k: {"ms": mean[k], "gbs": kb[k] / (mean[k] * 1e-3) / 1e9} for k in ("reduce", "state", "apply")}
-    dom = "apply"
-    roofline = {
-        "bound": "hbm", "kernel": "k_apply_dense", "achieved": kern[dom]["gbs"], "peak": peak,
-        "unit": "GB/s", "frac": kern[dom]["gbs"] / peak, "peak_kind": peak_kind,
-        "traffic": APPLY_TRAFFIC_BYTES.get(wl.name),
-        "algorithmic_bytes_per_launch": kb[dom],
-    }
-    if npan > 1:
-        # one apply launch per column panel: the figures are per pass
-        roofline["launches_per_pass"] = npan
+    # clocks sampled over every timed region of the run (the main step first)
+    with ClockSampler(local) as clocks:
+        barrier(world)
+        main = run_dense(wl, dev, args.steps, args.warmup, flush, seed=rank)
+        barrier(world)
+        ms = allreduce_max(world, main["ms_per_step"])
+        B = step_bytes(wl)
+        value = world * B / (ms * 1e-3) / 1e9
 
-    # end to end through the C ABI: the gradient comes in from pinned host
-    # memory, the step runs, and its result -- the optimizer state r, c
-    # (V + D floats) -- goes back to pinned host memory.  W stays on the
-    # device, as model weights do in training.
-    e2e = None
-    if not args.no_e2e:
-        n_e2e = max(1, min(args.steps, 10))
-        Gh = G.cpu().pin_memory()
-        Sh = torch.empty(emb.state.shape, dtype=emb.state.dtype, pin_memory=True)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        G2 = torch.empty_like(G)
-        ts = []
-        for _ in range(n_e2e):
-            t += 1
-            flush.zero_()
-            e0.record(stream)
-            G2.copy_(Gh, non_blocking=True)
-            emb.step_dense(W, G2, wl.lr, t)
-            Sh.copy_(emb.state, non_blocking=True)
-            e1.record(stream)
-            e1.synchronize()
-            ts.append(e0.elapsed_time(e1))
-        ms_copy = allreduce_max(world, sum(ts) / len(ts))
-        # the same, with the reduce pass reading G over the chip-to-chip link
-        # and staging it in HBM (ember_step_dense_from_host): no copy engine
-        ts = []
-        for _ in range(n_e2e):
-            t += 1
-            flush.zero_()
-            e0.record(stream)
-            emb.step_dense_from_host(W, Gh, G2, wl.lr, t)
-            Sh.copy_(emb.state, non_blocking=True)
-            e1.record(stream)
-            e1.synchronize()
-            ts.append(e0.elapsed_time(e1))
-        ms_e2e = allreduce_max(world, sum(ts) / len(ts))
-        e2e = {"value": world * B / (ms_e2e * 1e-3) / 1e9, "unit": "GB/s",
-               "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": emb.state.numel() * 4,
-               "ms_per_step": ms_e2e, "steps": n_e2e,
-               "what": "pinned-host G read by the reduce pass over the chip-to-chip link and staged in "
-                       "HBM (ember_step_dense_from_host), state r,c -> pinned host",
-               "copy_engine": {"ms_per_step": ms_copy, "value": world * B / (ms_copy * 1e-3) / 1e9,
-                               "what": "cudaMemcpyAsync of G to HBM, ember_step_dense, state back"}}
+        configs = {}
+        if not args.no_configs:
+            for tag, name, steps in CONFIGS:
+                cwl = synth.WORKLOADS[name]
+                if cwl.kind == "sparse":
+                    if args.no_sparse:
+                        continue
+                    configs[tag] = run_sparse(cwl, dev, max(2 * TRACE_EVERY, min(args.steps, steps)), args.warmup,
+                                              flush, seed=rank)
+                else:
+                    configs[tag] = run_dense(cwl, dev, max(2 * TRACE_EVERY, steps), args.warmup, flush, seed=rank)
+            configs["c5"] = {k: main[k] for k in ("workload", "ms_per_step", "value", "unit", "frac_of_measured_hbm",
+                                                 "launches_per_step", "roofline")}
+
+        # end to end through the C ABI: the gradient comes in from pinned host
+        # memory, the step runs, and its result -- the optimizer state r, c
+        # (V + D floats) -- goes back to pinned host memory.  W stays on the
+        # device, as model weights do in training.
+        e2e = None
+        if not args.no_e2e:
+            W = synth.init_weights(wl, rank, dev)
+            G = synth.dense_grad(wl, rank, 1, dev)
+            emb = Ember(wl.V, wl.D, wdtype=wl.wdtype, device=dev)
+            n_e2e = max(1, min(args.steps, 10))
+            Gh = G.cpu().pin_memory()
+            Sh = torch.empty(emb.state.shape, dtype=emb.state.dtype, pin_memory=True)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            G2 = torch.empty_like(G)
+            t = 0
+            ts = []
+            for _ in range(n_e2e):
+                t += 1
+                flush.zero_()
+                e0.record(stream)
+                G2.copy_(Gh, non_blocking=True)
+                emb.step_dense(W, G2, wl.lr, t)
+                Sh.copy_(emb.state, non_blocking=True)
+                e1.record(stream)
+                e1.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            ms_copy = allreduce_max(world, sum(ts) / len(ts))
+            # the same, with the reduce pass reading G over the chip-to-chip
+            # link and staging it in HBM (ember_step_dense_from_host)
+            ts = []
+            for _ in range(n_e2e):
+                t += 1
+                flush.zero_()
+                e0.record(stream)
+                emb.step_dense_from_host(W, Gh, G2, wl.lr, t)
+                Sh.copy_(emb.state, non_blocking=True)
+                e1.record(stream)
+                e1.synchronize()
+                ts.append(e0.elapsed_time(e1))
+            ms_e2e = allreduce_max(world, sum(ts) / len(ts))
+            if emb.device_status() != 0:
+                raise SystemExit("device status after the end-to-end steps")
+            e2e = {"value": world * B / (ms_e2e * 1e-3) / 1e9, "unit": "GB/s",
+                   "h2d_bytes_per_step": G.numel() * 4, "d2h_bytes_per_step": emb.state.numel() * 4,
+                   "ms_per_step": ms_e2e, "steps": n_e2e,
+                   "what": "pinned-host G read by the reduce pass over the chip-to-chip link and staged in "
+                           "HBM (ember_step_dense_from_host), state r,c -> pinned host",
+                   "copy_engine": {"ms_per_step": ms_copy, "value": world * B / (ms_copy * 1e-3) / 1e9,
+                                   "what": "cudaMemcpyAsync of G to HBM, ember_step_dense, state back"}}
+            del W, G, G2, emb, Gh
+
+        row_only = None
+        if not args.no_row_only:
+            Wr = synth.init_weights(wl, rank, dev)
+            Gr = synth.dense_grad(wl, rank, 1, dev)
+            row_only = run_row_only(wl, dev, max(2 * TRACE_EVERY, min(args.steps, 100)), args.warmup, flush, Wr, Gr)
+            row_only["frac_of_measured_hbm"] = row_only["value"] / peak
+            del Wr, Gr
+
+        lmhead = None
+        if not args.no_lmhead:
+            lwl = synth.WORKLOADS["lmhead_grad_v128256_d8192_t4096_bf16"]
+            lmhead = run_lmhead(lwl, dev, max(2 * TRACE_EVERY, min(args.steps, 20)), args.warmup, flush,
+                                seed=rank)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        import oracle
         rows = sample_rows_for(wl, 5.0)
         smp = OracleSample(wl, rows)
         secs = [smp.step() for _ in range(3)]
         sec = sum(secs) / len(secs)
+        cores = oracle.threads(host_cores())
+        rows_mc = sample_rows_for(wl, 5.0, all_cores=True)
+        smp_mc = OracleSample(wl, rows_mc)
+        smp_mc.step(all_cores=True)
+        secs_mc = [smp_mc.step(all_cores=True) for _ in range(3)]
+        sec_mc = sum(secs_mc) / len(secs_mc)
         cpu = {"value": smp.bytes / sec / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
                "sample": f"3 oracle dense steps on the first {rows} of {wl.V} rows (D={wl.D}), one thread",
-               "ms_per_step": sec * 1e3}
+               "ms_per_step": sec * 1e3,
+               "all_cores": {"value": smp_mc.bytes / sec_mc / 1e9, "unit": "GB/s", "cores": cores,
+                             "kind": "oracle (OpenMP build of the same source: the same bits)",
+                             "sample": f"3 oracle dense steps on the first {rows_mc} of {wl.V} rows "
+                                       f"(D={wl.D}), {cores} threads",
+                             "ms_per_step": sec_mc * 1e3}}
 
-    row_only = None
-    if not args.no_row_only:
-        row_only = run_row_only(wl, dev, max(2 * TRACE_EVERY, min(args.steps, 100)), args.warmup, flush, W, G)
-        row_only["frac_of_measured_hbm"] = row_only["value"] / peak
-
-    sparse = None
-    if not args.no_sparse:
-        swl = synth.WORKLOADS["sparse_v262144_d2048_bf16_n32768"]
-        sparse = run_sparse(swl, dev, max(2 * TRACE_EVERY, min(args.steps, 100)), args.warmup, flush,
-                            seed=rank)
-        sparse["frac_of_nominal_8TBs"] = sparse["value"] / NOMINAL_HBM_GBS
-        sparse["frac_of_measured_hbm"] = sparse["value"] / peak
-
-    lmhead = None
-    if not args.no_lmhead:
-        lwl = synth.WORKLOADS["lmhead_grad_v128256_d8192_t4096_bf16"]
-        lmhead = run_lmhead(lwl, dev, max(2 * TRACE_EVERY, min(args.steps, 20)), args.warmup, flush,
-                            seed=rank)
-
+    npan = main.get("roofline", {}).get("launches_per_pass", 1)
     line = {
         "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
@@ -657,19 +761,22 @@ def run_ours(args, world, rank, local):
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "w_dtype": wl.wdtype, "g_dtype": "f32",
                    "state_dtype": "f32", "l2": "flushed between steps (512 MiB write, outside the events)",
                    "parallelism": f"replicas x{world}"},
-        "roofline": roofline,
+        "roofline": main["roofline"],
         "cpu_baseline": cpu,
         "e2e": e2e,
-        "gpu_launches": (2 * npan + 1) * args.steps,
+        "gpu_launches": main["gpu_launches"],
         "clocks": clocks.summary(),
         "params_per_s": world * wl.V * wl.D / (ms * 1e-3),
         "frac_of_nominal_8TBs": value / world / NOMINAL_HBM_GBS,
         "frac_of_measured_hbm": value / world / peak,
-        "kernels": kern,
-        "ms_per_step_traced": mean["traced_step"],
-        "timing": f"step time: CUDA events around each untraced step; kernel times: every {TRACE_EVERY}th step records events at kernel boundaries",
-        "wall_s_timed_region": wall,
-        "sparse": sparse,
+        "peak_kind": peak_kind,
+        "kernels": main.get("kernels"),
+        "ms_per_step_traced": main.get("ms_per_step_traced"),
+        "timing": main["timing"],
+        "wall_s_timed_region": main["wall_s_timed_region"],
+        "column_panels": npan,
+        "configs": configs,
+        "sparse": configs.get("c4"),
         "row_only": row_only,
         "lmhead_fused": lmhead,
     }
@@ -690,6 +797,7 @@ def main():
     ap.add_argument("--no-sparse", action="store_true")
     ap.add_argument("--no-row-only", action="store_true")
     ap.add_argument("--no-lmhead", action="store_true")
+    ap.add_argument("--no-configs", action="store_true")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

@@ -122,6 +122,13 @@ void ember_destroy(ember_handle *h);
  * NULL handle. */
 int ember_column_panels(const ember_handle *h, int vector_path);
 
+/* Kernel launches one ember_step_dense of this handle makes without trace
+ * events: 1 for a small table (one cluster launch), 2 for the row-only
+ * variant (its one-pass kernel and the column state), otherwise 2 per
+ * column panel plus the state pass.  vector_path as for
+ * ember_column_panels.  Host only; 0 for a NULL handle. */
+int ember_dense_step_launches(const ember_handle *h, int vector_path);
+
 /* Number of fp32 values of optimizer state: exactly V + D (Algorithm 1
  * keeps r in R^V and c in R^D).  The caller's state buffer holds r in
  * [0, V) followed by c in [V, V + D).  A new table starts from all zeros

@@ -30,28 +30,44 @@ _VARIANTS = {"full": 0, "row": 1, "col": 2}
 _lib = None
 
 
+_lib_omp = None
+
+
 def _load():
     global _lib
     if _lib is None:
         # EMBER_ORACLE_LIB lets the mutation test load a deliberately broken copy.
-        lib = ctypes.CDLL(os.environ.get("EMBER_ORACLE_LIB") or build_oracle())
-        i64, dbl, vp, ip = ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_int
-        lib.ember_oracle_step_dense.argtypes = [
-            i64, i64, ip, vp, vp, vp, vp, dbl, i64, dbl, dbl, ip, ip, ip, vp]
-        lib.ember_oracle_step_dense.restype = ip
-        lib.ember_oracle_step_sparse.argtypes = [
-            i64, i64, ip, vp, i64, vp, vp, vp, vp, dbl, i64, dbl, dbl, ip, ip, ip, vp]
-        lib.ember_oracle_step_sparse.restype = ip
-        lib.ember_oracle_dedup.argtypes = [i64, vp, i64, vp, vp]
-        lib.ember_oracle_dedup.restype = i64
-        lib.ember_oracle_round_bf16.argtypes = [i64, vp, vp]
-        lib.ember_oracle_round_bf16.restype = None
-        lib.ember_oracle_bf16_to_double.argtypes = [i64, vp, vp]
-        lib.ember_oracle_bf16_to_double.restype = None
-        lib.ember_oracle_lmhead_grad.argtypes = [i64, i64, i64, vp, vp, i64, vp, vp, vp]
-        lib.ember_oracle_lmhead_grad.restype = ip
-        _lib = lib
+        _lib = _bind(ctypes.CDLL(os.environ.get("EMBER_ORACLE_LIB") or build_oracle()))
     return _lib
+
+
+def _load_omp():
+    """The same source built with -fopenmp (for the all-cores CPU baseline)."""
+    global _lib_omp
+    if _lib_omp is None:
+        _lib_omp = _bind(ctypes.CDLL(build_oracle(openmp=True)))
+    return _lib_omp
+
+
+def _bind(lib):
+    i64, dbl, vp, ip = ctypes.c_int64, ctypes.c_double, ctypes.c_void_p, ctypes.c_int
+    lib.ember_oracle_step_dense.argtypes = [
+        i64, i64, ip, vp, vp, vp, vp, dbl, i64, dbl, dbl, ip, ip, ip, vp]
+    lib.ember_oracle_step_dense.restype = ip
+    lib.ember_oracle_step_sparse.argtypes = [
+        i64, i64, ip, vp, i64, vp, vp, vp, vp, dbl, i64, dbl, dbl, ip, ip, ip, vp]
+    lib.ember_oracle_step_sparse.restype = ip
+    lib.ember_oracle_dedup.argtypes = [i64, vp, i64, vp, vp]
+    lib.ember_oracle_dedup.restype = i64
+    lib.ember_oracle_round_bf16.argtypes = [i64, vp, vp]
+    lib.ember_oracle_round_bf16.restype = None
+    lib.ember_oracle_bf16_to_double.argtypes = [i64, vp, vp]
+    lib.ember_oracle_bf16_to_double.restype = None
+    lib.ember_oracle_lmhead_grad.argtypes = [i64, i64, i64, vp, vp, i64, vp, vp, vp]
+    lib.ember_oracle_lmhead_grad.restype = ip
+    lib.ember_oracle_threads.argtypes = [ip]
+    lib.ember_oracle_threads.restype = ip
+    return lib
 
 
 def _ptr(a):
@@ -77,16 +93,24 @@ def _diag(d):
     return {"bc": d[0], "rbar": d[1], "cbar": d[2], "s": d[3], "zero_rows": int(d[4])}
 
 
+def threads(n=0):
+    """Threads of the all-cores build: n > 0 sets the count; returns it."""
+    return _load_omp().ember_oracle_threads(int(n))
+
+
 def step_dense(W, G, r, c, lr, t, beta2=0.999, eps=1e-8, maximize=False,
-               bias_correction=True, variant="full"):
+               bias_correction=True, variant="full", all_cores=False):
     """One dense Ember step (Algorithm 1) in place on W, r, c; returns the
-    step's scalars (1-beta2^t, mean rhat, mean chat, s, zero rows)."""
+    step's scalars (1-beta2^t, mean rhat, mean chat, s, zero rows).
+    all_cores=True runs the OpenMP build of the same source (see threads());
+    it gives the same bits."""
     V, D = _check_state(W, r, c)
     G = np.ascontiguousarray(G, dtype=np.float32)
     if G.shape != (V, D):
         raise ValueError("G must have W's shape")
     d = np.zeros(5, np.float64)
-    rc = _load().ember_oracle_step_dense(
+    lib = _load_omp() if all_cores else _load()
+    rc = lib.ember_oracle_step_dense(
         V, D, int(W.dtype == np.uint16), _ptr(W), _ptr(G), _ptr(r), _ptr(c),
         float(lr), int(t), float(beta2), float(eps), int(bool(maximize)),
         int(bool(bias_correction)), _VARIANTS[variant], _ptr(d))

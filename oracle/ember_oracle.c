@@ -38,16 +38,25 @@
  *     rhat = r, chat = c (the bias-correction ablation of the appendix).
  *
  * Built with gcc -O2 -fno-fast-math -ffp-contract=off so that every
- * operation rounds exactly as written.
+ * operation rounds exactly as written.  The timed CPU baseline also builds
+ * it with -fopenmp: the row loops and the blocks of the column loop then run
+ * on all host cores, and since every sum keeps its order (each row's sum
+ * over its columns, each column's sum over the rows in index order) that
+ * build gives the same bits.
  */
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
 #include <string.h>
+#ifdef _OPENMP
+#include <omp.h>
+#endif
 
 #define ORC_FULL 0
 #define ORC_ROW 1
 #define ORC_COL 2
+
+#define ORC_COL_BLOCK 64 /* columns per block of the column-sum loop */
 
 #define ORC_OK 0
 #define ORC_EINVAL -1
@@ -143,6 +152,7 @@ static int alg1_step(int64_t V, int64_t D, int w_is_bf16, void *W,
         return ORC_EINVAL;
 
     /* Row second moment: r_i <- beta2 r_i + (1-beta2) mean_j g_ij^2. */
+    #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < V; ++i) {
         double sum = 0.0;
         for (int64_t j = 0; j < D; ++j) {
@@ -157,11 +167,17 @@ static int alg1_step(int64_t V, int64_t D, int w_is_bf16, void *W,
     double *colsum = (double *)calloc((size_t)D, sizeof(double));
     if (!colsum)
         return ORC_ENOMEM;
-    for (int64_t i = 0; i < V; ++i)
-        for (int64_t j = 0; j < D; ++j) {
-            double g = grad_at(Gf, Gd, i * D + j);
-            colsum[j] += g * g;
-        }
+    /* Each column's sum runs over the rows in index order; the columns are
+       independent, so they are taken in blocks (in parallel under OpenMP). */
+    #pragma omp parallel for schedule(static)
+    for (int64_t jb = 0; jb < D; jb += ORC_COL_BLOCK) {
+        int64_t je = (jb + ORC_COL_BLOCK < D) ? jb + ORC_COL_BLOCK : D;
+        for (int64_t i = 0; i < V; ++i)
+            for (int64_t j = jb; j < je; ++j) {
+                double g = grad_at(Gf, Gd, i * D + j);
+                colsum[j] += g * g;
+            }
+    }
     for (int64_t j = 0; j < D; ++j) {
         double mean_col = colsum[j] / (double)V;
         c[j] = (float)(beta2 * (double)c[j] + (1.0 - beta2) * mean_col);
@@ -185,6 +201,7 @@ static int alg1_step(int64_t V, int64_t D, int w_is_bf16, void *W,
     double s = sqrt(rbar * cbar);
 
     /* Preconditioner vtil = rhat chat^T / s, never stored; update. */
+    #pragma omp parallel for schedule(static)
     for (int64_t i = 0; i < V; ++i) {
         double rhat = (double)r[i] / bc;
         for (int64_t j = 0; j < D; ++j) {
@@ -223,6 +240,20 @@ int ember_oracle_step_dense(int64_t V, int64_t D, int w_is_bf16, void *W,
         return ORC_EINVAL;
     return alg1_step(V, D, w_is_bf16, W, G, NULL, r, c, lr, t, beta2, eps,
                      maximize, bias_correction, variant, diag);
+}
+
+/* Threads of the OpenMP build: n > 0 sets the count; returns the count in
+ * use (always 1 in the plain build). */
+int ember_oracle_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0)
+        omp_set_num_threads(n);
+    return omp_get_max_threads();
+#else
+    (void)n;
+    return 1;
+#endif
 }
 
 /* ------------------------------------------------------------------ */

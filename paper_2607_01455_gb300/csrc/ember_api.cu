@@ -123,6 +123,13 @@ int ember_column_panels(const ember_handle *h, int vector_path)
     return m.npanels;
 }
 
+int ember_dense_step_launches(const ember_handle *h, int vector_path)
+{
+    if (!h)
+        return 0;
+    return dense_step_launches(h->V, h->D, h->wdtype == EMBER_BF16, h->hp.variant, vector_path != 0);
+}
+
 size_t ember_state_numel(const ember_handle *h)
 {
     return h ? (size_t)(h->V + h->D) : 0;

@@ -761,20 +761,54 @@ struct SmallArgs {
     int variant;
 };
 
-constexpr int kMaxClusterCtas = 8;
-constexpr size_t kSmallSmemMax = 200 << 10;
 
-// Shared memory of k_dense_cluster, in bytes from the dynamic base: kept G,
-// kept W, then D floats each of the column partial, the combine buffer, the
-// old c, the new c (then the column scales), and ceil(D/32) floats.
+// Shared memory of k_dense_cluster, from the dynamic base: kept G, kept W
+// (one 16- or 8-byte slot per thread, per row and access of each reduce
+// iteration), then D floats each of the column partial, the combine buffer,
+// the old c, the new c (then the column scales), and ceil(D/32) floats.
 template <int CPT, int R, bool BF16>
 __host__ __device__ constexpr size_t small_slots(int nits) { return (size_t)nits * R * CPT * kThreads; }
-template <int CPT, int R, bool BF16>
-__host__ __device__ constexpr size_t small_smem_bytes(int nits, int D)
+
+}  // namespace
+
+// Whether a dense step of this table runs as one cluster launch: the vector
+// path, one column panel, at most kMaxClusterCtas CTAs, and the kept G and W
+// (every slot of the CTA's reduce iterations) within kSmallSmemMax of shared
+// memory.  *nits: reduce iterations per CTA; *smem: dynamic shared memory.
+bool small_table_plan(int64_t V, int64_t D, bool wbf16, const ColMap &m, int *nits, size_t *smem)
 {
-    return small_slots<CPT, R, BF16>(nits) * (16 + (BF16 ? 8 : 16)) + (size_t)4 * D * sizeof(float) +
-           (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float);
+    const int nparts = dense_parts(V, D);
+    if (m.vec != 4 || m.npanels != 1 || nparts > kMaxClusterCtas)
+        return false;
+    const int R1 = (16 / m.cpt) < 1 ? 1 : (16 / m.cpt);
+    const int rows_per_it = (kThreads / m.tpr) * R1;
+    const int64_t rows = (V + nparts - 1) / nparts;
+    const int64_t n = (rows + rows_per_it - 1) / rows_per_it;
+    const size_t slots = (size_t)n * R1 * m.cpt * kThreads;
+    const size_t bytes = slots * (16 + (wbf16 ? 8 : 16)) + (size_t)4 * D * sizeof(float) +
+                         (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float);
+    if (bytes > kSmallSmemMax)
+        return false;
+    *nits = (int)n;
+    *smem = bytes;
+    return true;
 }
+
+int dense_step_launches(int64_t V, int64_t D, bool wbf16, int variant, bool vec4)
+{
+    ColMap m;
+    if (!choose_colmap(D, vec4, &m))
+        return 0;
+    int nits = 0;
+    size_t sm = 0;
+    if (m.npanels == 1 && variant == EMBER_VARIANT_ROW)
+        return 2;  // the one-pass row-only kernel and the column state
+    if (variant != EMBER_VARIANT_ROW && small_table_plan(V, D, wbf16, m, &nits, &sm))
+        return 1;
+    return 2 * m.npanels + 1;
+}
+
+namespace {
 
 template <int CPT, int R, bool BF16>
 __global__ void __launch_bounds__(kThreads, 1)
@@ -1283,35 +1317,30 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         return cudaGetLastError();
     }
     if constexpr (VEC == 4) {
-        if (!a.lm && !a.G_stage && !a.trace && np == 1 && nparts <= kMaxClusterCtas) {
-            // a small table: the whole step in one cluster launch, when the
-            // kept G and W fit shared memory
-            const int64_t rows = (a.V + nparts - 1) / nparts;
-            const int rows_per_it = rg * R1;
-            const int nits = (int)((rows + rows_per_it - 1) / rows_per_it);
-            const size_t sm = a.wbf16 ? small_smem_bytes<CPT, R1, true>(nits, D)
-                                      : small_smem_bytes<CPT, R1, false>(nits, D);
-            if (sm <= kSmallSmemMax) {
-                auto *k = a.wbf16 ? k_dense_cluster<CPT, R1, true> : k_dense_cluster<CPT, R1, false>;
-                e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
-                if (e != cudaSuccess)
-                    return e;
-                SmallArgs sa{a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, nits, kc, a.eps, a.lr_signed, a.variant};
-                cudaLaunchConfig_t cfg = {};
-                cfg.gridDim = dim3(nparts);
-                cfg.blockDim = dim3(kThreads);
-                cfg.dynamicSmemBytes = sm;
-                cfg.stream = a.stream;
-                cudaLaunchAttribute attr[1];
-                attr[0].id = cudaLaunchAttributeClusterDimension;
-                attr[0].val.clusterDim.x = nparts;
-                attr[0].val.clusterDim.y = 1;
-                attr[0].val.clusterDim.z = 1;
-                cfg.attrs = attr;
-                cfg.numAttrs = 1;
-                e = cudaLaunchKernelEx(&cfg, k, sa);
-                return e != cudaSuccess ? e : cudaGetLastError();
-            }
+        int nits = 0;
+        size_t sm = 0;
+        if (!a.lm && !a.G_stage && !a.trace && small_table_plan(a.V, a.D, a.wbf16 != 0, a.map, &nits, &sm)) {
+            // a small table: the whole step in one cluster launch, the kept
+            // G and W in shared memory
+            auto *k = a.wbf16 ? k_dense_cluster<CPT, R1, true> : k_dense_cluster<CPT, R1, false>;
+            e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e != cudaSuccess)
+                return e;
+            SmallArgs sa{a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, nits, kc, a.eps, a.lr_signed, a.variant};
+            cudaLaunchConfig_t cfg = {};
+            cfg.gridDim = dim3(nparts);
+            cfg.blockDim = dim3(kThreads);
+            cfg.dynamicSmemBytes = sm;
+            cfg.stream = a.stream;
+            cudaLaunchAttribute attr[1];
+            attr[0].id = cudaLaunchAttributeClusterDimension;
+            attr[0].val.clusterDim.x = nparts;
+            attr[0].val.clusterDim.y = 1;
+            attr[0].val.clusterDim.z = 1;
+            cfg.attrs = attr;
+            cfg.numAttrs = 1;
+            e = cudaLaunchKernelEx(&cfg, k, sa);
+            return e != cudaSuccess ? e : cudaGetLastError();
         }
     }
     if (a.lm) {

@@ -111,6 +111,13 @@ struct ColMap {
 
 bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m);
 
+// Small tables run the whole dense step as one thread-block cluster launch
+// (see ember_dense.cu); the plan and the launch count of a dense step.
+constexpr int kMaxClusterCtas = 8;
+constexpr size_t kSmallSmemMax = 200 << 10;
+bool small_table_plan(int64_t V, int64_t D, bool wbf16, const ColMap &m, int *nits, size_t *smem);
+int dense_step_launches(int64_t V, int64_t D, bool wbf16, int variant, bool vec4);
+
 // LM-head gradient G = dlogits^T hidden (T tokens, bf16 inputs, fp32 G).
 struct LmArgs {
     int64_t V, D, T;

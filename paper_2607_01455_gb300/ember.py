@@ -41,6 +41,7 @@ EXPORTS = (
     "ember_lmhead_grad", "ember_step_lmhead",
     "ember_shard_rows", "ember_shard_scale_bytes", "ember_shard_exchange_bytes", "ember_shard_reduce",
     "ember_shard_pack", "ember_shard_update", "ember_column_panels", "ember_set_wait_limit_ns",
+    "ember_dense_step_launches",
 )
 
 
@@ -96,6 +97,7 @@ def lib():
             "ember_shard_pack": (st, [vp, ip, ip, vp, vp, vp]),
             "ember_shard_update": (st, [vp, ip, ip, vp, vp, vp, vp, vp, flt, i64, vp]),
             "ember_column_panels": (ip, [vp, ip]),
+            "ember_dense_step_launches": (ip, [vp, ip]),
             "ember_set_wait_limit_ns": (st, [vp, ctypes.c_uint64]),
         }
         for name, (res, args) in sig.items():
@@ -140,6 +142,11 @@ def ember_column_panels(h, vector_path=True):
     """Column panels a step of this handle runs in (1 unless D is wider than
     one CTA's row)."""
     return lib().ember_column_panels(h, int(bool(vector_path)))
+
+
+def ember_dense_step_launches(h, vector_path=True):
+    """Kernel launches of one ember_step_dense of this handle (1 for a small table)."""
+    return lib().ember_dense_step_launches(h, int(bool(vector_path)))
 
 
 def ember_hparams_default():
@@ -356,6 +363,9 @@ class Ember:
 
     def column_panels(self, vector_path=True):
         return ember_column_panels(self.handle, vector_path)
+
+    def dense_step_launches(self, vector_path=True):
+        return ember_dense_step_launches(self.handle, vector_path)
 
     def trace(self, events):
         ember_set_trace_events(self.handle, events)

@@ -15,14 +15,18 @@ where the new weight nearly cancels to zero, is then far above 1e-5 lr; the
 floor therefore also takes the oracle's own step |W_t - W_{t-1}| when the
 previous weights are given.
 
-One refinement of the bf16 bar, derived from the arithmetic: the kernel forms
-W - lr u in fp32 (the paper fixes no precision), so u carries a relative
-error of a few fp32 ulps (~3e-7).  Where the new weight nearly cancels to
-zero, a bf16 ulp of the result is smaller than that error (|W_new| below
-~4e-7 for |W| ~ 0.02), and no fp32 computation can promise 1 ulp there.
-Those elements are held to the fp32-weight bar instead: |got - want| <=
-1e-5 max(|want|, lr).  The share of elements that pass only that way is
-returned so that the tests can bound it.
+One refinement of the bf16 bar, derived from the arithmetic: the kernel
+forms W - lr u in fp32 (the paper fixes no precision), so the new weight
+carries an error of a few fp32 ulps of the step |W_t - W_{t-1}| (about
+4 * 2^-24 of it).  Rounding to bf16 can then land more than one bf16 ulp
+(2^-8 of |W_t|) away from the oracle's rounding only where that error
+exceeds a bf16 ulp of the result, i.e. where the step nearly cancels the
+weight: |W_t| < 2^-14 |W_t - W_{t-1}|.  Every element more than 1 ulp apart
+must lie in that set (with a margin: |W_t| <= 2^-12 of the step, or of lr
+when the previous weights are not given) and meet the fp32-weight bar
+|got - want| <= 1e-5 max(|want|, lr, step).  There is no count cap: the
+condition is the bar.  The share of such elements is returned and collected
+for the test summary.
 """
 import numpy as np
 import torch
@@ -50,28 +54,50 @@ def bf16_ulp_distance(a, b):
     return np.abs(bf16_ordinal(a) - bf16_ordinal(b))
 
 
-def check_weights(got, want, lr, what="W", prev=None):
+# largest share of bf16 elements more than 1 ulp apart seen by any check
+# (reported in the test session's summary)
+OBSERVED = {"frac_beyond_1ulp": 0.0, "checks": 0}
+
+
+def check_weights(got, want, lr, what="W", prev=None, record=False, summed_input=False):
     """`prev`: the weights before the step (same dtype), whose difference from
-    `want` is the oracle's own step size."""
+    `want` is the oracle's own step size.  record: count this check in the
+    session summary (the gated GPU steps do).  summed_input: the GPU formed
+    the gradient itself in fp32 (the sparse step's per-id sums, whose error
+    is absolute, about 2^-22 of the sum of the summed rows' magnitudes): an
+    element whose sum nearly cancels then carries a relative error the
+    oracle's fp64 sum does not, so outside the cancellation set up to
+    max(2, 1e-5 of the elements) may also differ by more than 1 ulp, within
+    the fp32-weight bar."""
     if got.dtype == np.uint16:
         d = bf16_ulp_distance(got, want)
         far = d > BF16_ULPS
         n_far = int(far.sum())
         if n_far:
-            assert n_far <= max(2, 1e-3 * d.size), f"{what}: {n_far} elements more than 1 bf16 ulp apart"
             g = oracle.bf16_to_float64(got[far])
             w = oracle.bf16_to_float64(want[far])
-            floor = np.maximum(np.abs(w), abs(lr))
-            if prev is not None:
-                floor = np.maximum(floor, np.abs(w - oracle.bf16_to_float64(prev[far])))
+            step = np.abs(w - oracle.bf16_to_float64(prev[far])) if prev is not None else np.full(w.shape, abs(lr))
+            near = np.abs(w) <= 2.0 ** -12 * step
+            n_other = int((~near).sum())
+            k = int(np.argmin(near)) if not near.all() else 0
+            allowed = max(2, int(1e-5 * d.size)) if summed_input else 0
+            assert n_other <= allowed, (
+                f"{what}: {n_other} elements more than 1 bf16 ulp apart where the step does not cancel the "
+                f"weight (at most {allowed} allowed), e.g. {int(d[far][k])} ulps: {g[k]!r} vs {w[k]!r} "
+                f"(step {step[k]:.3g})")
+            floor = np.maximum(np.maximum(np.abs(w), abs(lr)), step)
             rel = np.abs(g - w) / floor
             k = int(rel.argmax())
             assert rel[k] <= REL_TOL, (
                 f"{what}: {int(d.max())} bf16 ulps apart, {g[k]!r} vs {w[k]!r} "
-                f"(relative {rel[k]:.3g} of max(|W|, lr))")
+                f"(relative {rel[k]:.3g} of max(|W|, lr, step))")
+        frac = n_far / max(d.size, 1)
+        if record:
+            OBSERVED["frac_beyond_1ulp"] = max(OBSERVED["frac_beyond_1ulp"], frac)
+            OBSERVED["checks"] += 1
         return {"max_ulp": int(d.max()) if d.size else 0,
                 "frac_differ": float((d > 0).mean()) if d.size else 0.0,
-                "frac_near_zero_fallback": n_far / max(d.size, 1)}
+                "frac_near_zero_fallback": frac}
     g = got.astype(np.float64)
     w = want.astype(np.float64)
     floor = np.maximum(np.abs(w), abs(lr))
@@ -107,9 +133,10 @@ class Opt:
         self.bias_correction, self.variant = bias_correction, variant
 
 
-def gated_dense_step(emb, W, G, lr, t, opt):
+def gated_dense_step(emb, W, G, lr, t, opt, all_cores=False):
     """Run one GPU step and the oracle's step from the same W_{t-1}, state_{t-1}
-    and G; compare W_t and the state.  Returns error statistics."""
+    and G; compare W_t and the state.  Returns error statistics.  all_cores
+    runs the oracle's OpenMP build (the same bits; for the largest tables)."""
     V = emb.V
     W0 = w_to_host(W)
     st0 = emb.state.cpu().numpy().copy()
@@ -118,10 +145,10 @@ def gated_dense_step(emb, W, G, lr, t, opt):
     torch.cuda.synchronize()
     r, c = st0[:V].copy(), st0[V:].copy()
     Wo = W0.copy()
-    oracle.step_dense(Wo, Gh, r, c, float(np.float32(lr)), t, **oracle_kwargs(opt))
+    oracle.step_dense(Wo, Gh, r, c, float(np.float32(lr)), t, all_cores=all_cores, **oracle_kwargs(opt))
     st = emb.state.cpu().numpy()
     stats = {}
     stats["r"] = check_state(st[:V], r, "r")
     stats["c"] = check_state(st[V:], c, "c")
-    stats["W"] = check_weights(w_to_host(W), Wo, lr, prev=W0)
+    stats["W"] = check_weights(w_to_host(W), Wo, lr, prev=W0, record=True)
     return stats

@@ -105,7 +105,7 @@ def _run_workload(cuda_device, name, gate_steps, steps=None):
     for t in range(1, last + 1):
         synth.dense_grad(wl, 0, t, cuda_device, out=G, scales=scales, sets=sets)
         if t in gate_steps:
-            gated_dense_step(emb, W, G, wl.lr, t, Opt())
+            gated_dense_step(emb, W, G, wl.lr, t, Opt(), all_cores=True)
         else:
             emb.step_dense(W, G, wl.lr, t)
     torch.cuda.synchronize()
@@ -127,8 +127,9 @@ def test_dense_workload_tied_151936x896(cuda_device):
 
 
 def test_dense_workload_lmhead_128256x8192(cuda_device):
-    """The large LM head in the launch configuration the benchmark times."""
-    _run_workload(cuda_device, "dense_lmhead_v128256_d8192_bf16", {1, 2, 50})
+    """The large LM head in the launch configuration the benchmark times,
+    gated at steps 1, 2, 3, 10, 20, 30, 40 and 50."""
+    _run_workload(cuda_device, "dense_lmhead_v128256_d8192_bf16", {1, 2, 3, 10, 20, 30, 40, 50})
 
 
 def test_dense_deterministic_and_resumable(cuda_device):

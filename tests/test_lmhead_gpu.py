@@ -112,7 +112,7 @@ def test_step_lmhead_gated(cuda_device, V, D, T, wdtype):
         st = emb.state.cpu().numpy()
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
-        check_weights(w_to_host(W), Wo, 1e-3, prev=W0)
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0, record=True)
 
 
 @pytest.mark.parametrize("opt", [Opt(variant="row"), Opt(variant="col"), Opt(maximize=True),
@@ -130,11 +130,12 @@ def test_step_lmhead_hyperparameters(cuda_device, opt):
         emb.step_lmhead(W, dl, h, G, 1e-3, t)
         torch.cuda.synchronize()
         r, c = st0[:V].copy(), st0[V:].copy()
-        oracle.step_dense(W0, G.cpu().numpy(), r, c, float(np.float32(1e-3)), t, **oracle_kwargs(opt))
+        Wo = W0.copy()
+        oracle.step_dense(Wo, G.cpu().numpy(), r, c, float(np.float32(1e-3)), t, **oracle_kwargs(opt))
         st = emb.state.cpu().numpy()
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
-        check_weights(w_to_host(W), W0, 1e-3)
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0, record=True)
 
 
 def test_step_lmhead_writes_the_same_G_and_is_deterministic(cuda_device):
@@ -273,4 +274,4 @@ def test_bounded_wait_gives_up_and_the_next_step_recovers(cuda_device):
         st = emb.state.cpu().numpy()
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
-        check_weights(w_to_host(W), Wo, 1e-3, prev=W0)
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0, record=True)

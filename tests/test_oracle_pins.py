@@ -522,3 +522,25 @@ def test_lmhead_grad_roles_of_the_factors_and_row_selection():
     # matmul of the exact factors in fp64 agrees to rounding
     ref = oracle.bf16_to_float64(dl).T @ oracle.bf16_to_float64(hd)
     np.testing.assert_allclose(G, ref, rtol=0, atol=1e-12 * np.abs(ref).max())
+
+
+def test_all_cores_build_gives_the_same_bits():
+    """The CPU baseline's OpenMP build of the oracle splits only independent
+    loops (rows; blocks of columns, each column still summed over the rows in
+    index order), so it must reproduce the plain build bit for bit."""
+    rng = np.random.default_rng(11)
+    V, D = 517, 203
+    W0 = (rng.standard_normal((V, D)) * 0.02).astype(np.float32)
+    Gs = [(rng.standard_normal((V, D)) * 1e-3).astype(np.float32) for _ in range(3)]
+    assert oracle.threads(4) >= 1
+    outs = []
+    for all_cores in (False, True):
+        Wf, Wh = W0.copy(), oracle.round_bf16(W0.astype(np.float64))
+        r1, c1 = np.zeros(V, np.float32), np.zeros(D, np.float32)
+        r2, c2 = np.zeros(V, np.float32), np.zeros(D, np.float32)
+        for t, G in enumerate(Gs, start=1):
+            oracle.step_dense(Wf, G, r1, c1, 1e-3, t, all_cores=all_cores)
+            oracle.step_dense(Wh, G, r2, c2, 1e-3, t, variant="col", all_cores=all_cores)
+        outs.append((Wf, Wh, r1, c1, r2, c2))
+    for a, b in zip(*outs):
+        assert np.array_equal(a, b)

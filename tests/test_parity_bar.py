@@ -62,3 +62,25 @@ def test_bf16_near_cancellation_uses_the_step_floor():
     far[1] += 2
     with pytest.raises(AssertionError):
         check_weights(far, want, lr, prev=prev)
+
+
+def test_bf16_beyond_one_ulp_only_where_the_step_cancels_the_weight():
+    """Two ulps off on a small weight that the step does not cancel fails,
+    however few such elements there are: the near-cancellation set
+    (|W_t| <= 2^-12 of the step) is the only place a correct fp32 update can
+    land more than one bf16 ulp from the oracle."""
+    import oracle
+    lr = 1e-3
+    prev = oracle.round_bf16(np.full(100000, 0.02))
+    want = oracle.round_bf16(np.concatenate([[2e-5], np.full(99999, 0.019)]))
+    got = want.copy()
+    got[0] += 2  # |W_t| = 2e-5 against a 0.02 step: 1e-3 of it, not cancelling
+    with pytest.raises(AssertionError):
+        check_weights(got, want, lr, prev=prev)
+    want[0] = oracle.round_bf16(np.array([6e-6]))[0]  # 3e-4 of the step: still outside 2^-12
+    got[0] = want[0] + 2
+    with pytest.raises(AssertionError):
+        check_weights(got, want, lr, prev=prev)
+    want[0] = oracle.round_bf16(np.array([4e-7]))[0]  # 2e-5 of the step: inside 2^-12
+    got[0] = want[0] + 2
+    check_weights(got, want, lr, prev=prev)

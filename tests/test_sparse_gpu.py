@@ -51,7 +51,7 @@ def gated_sparse_step(emb, W, ids, rows, lr, t, opt):
     check_state(st[:V], r, "r")
     check_state(st[V:], c, "c")
     Wg = w_to_host(W)
-    check_weights(Wg, Wo, lr, prev=W0)
+    check_weights(Wg, Wo, lr, prev=W0, record=True, summed_input=True)
     # rows whose id does not occur keep their weights bit for bit
     touched = np.zeros(V, bool)
     ids_h = ids.cpu().numpy().astype(np.int64)
@@ -133,7 +133,7 @@ def test_sparse_equals_dense_on_scatter_summed_gradient(cuda_device):
         ed.step_dense(Wd, G.float(), 1e-3, t)
         torch.cuda.synchronize()
         check_state(es.state.cpu().numpy(), ed.state.cpu().numpy(), "state")
-        check_weights(w_to_host(Ws), w_to_host(Wd), 1e-3)
+        check_weights(w_to_host(Ws), w_to_host(Wd), 1e-3, summed_input=True)
 
 
 def test_sparse_edge_cases(cuda_device):

@@ -158,7 +158,7 @@ def test_wide_sparse_parity(cuda_device, V, D, N):
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
         Wg = w_to_host(W)
-        check_weights(Wg, Wo, 1e-3, prev=W0)
+        check_weights(Wg, Wo, 1e-3, prev=W0, record=True, summed_input=True)
         touched = np.zeros(V, bool)
         touched[ids.cpu().numpy()] = True
         assert np.array_equal(Wg[~touched], W0[~touched])
@@ -189,7 +189,7 @@ def test_wide_step_lmhead_gated(cuda_device, V, D, T):
         st = emb.state.cpu().numpy()
         check_state(st[:V], r, "r")
         check_state(st[V:], c, "c")
-        check_weights(w_to_host(W), Wo, 1e-3, prev=W0)
+        check_weights(w_to_host(W), Wo, 1e-3, prev=W0, record=True)
 
 
 def test_wide_tables_are_refused_by_shards_and_noalloc(cuda_device):
