@@ -67,17 +67,6 @@ namespace {
 
 using namespace dev;
 
-// beta2 r + (1 - beta2) m in fp32 with the coefficients carried as float
-// pairs (StepConsts): within about an ulp of the fp64 value, and the fixed
-// point stays at r = m, which rounding beta2 and 1 - beta2 to single floats
-// would shift by about 1e-5 of r at beta2 = 0.999.  With m = 0 (a row outside
-// a sparse batch) it is the correctly rounded product beta2 r in all but
-// near-tie cases.
-__device__ __forceinline__ float ema_pair(const EmaPair &e, float r, float m)
-{
-    return fmaf(e.bh, r, fmaf(e.bl, r, fmaf(e.ah, m, e.al * m)));
-}
-
 // ---------------------------------------------------------------------------
 // Reduce: one read of G.  VEC columns per access, CPT accesses per thread per
 // row, R rows per row group per iteration.  The CTA's rows are those of CTA
@@ -351,10 +340,10 @@ struct ColSource {
 };
 
 constexpr int kStateWarps = kStateThreads / 32;
-// partial rows per warp held in registers by the column pass (304 rows of
-// the dense step fit; more, as the LM-head and sparse steps have, take two
-// passes through L2)
-constexpr int kRegParts = 38;
+// partial rows per warp held in registers by the column pass (the dense
+// step's 304 and the sparse step's 456 rows fit; more, as the LM-head step
+// has, take two passes through L2)
+constexpr int kRegParts = 64;
 static_assert(kRegParts * kStateWarps >= kGridCtas, "the dense step's partial rows fit the register path");
 
 __device__ __forceinline__ void column_group(const ColSource &src, int group, float *__restrict__ c,
@@ -558,11 +547,13 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r, float *__rest
 // sum of r over the table is the exact fixed-point total of the nrsum per-CTA
 // sums, or, in a row-sharded step, comes with the exchanged totals.
 struct RowPass {
-    float *r;               // r[V], updated (sparse step only)
-    int32_t *slot;          // touched-row map, cleared here
-    const float *rowpart;   // per (distinct id, slice) sums of g^2
+    float *r;               // r[V], updated
+    int32_t *slot;          // sparse step: touched-row map, cleared here
+    const float *rowpart;   // per (distinct id, slice) sums of g^2, or per (slice, row)
     int nslices;
     int nrow_ctas;          // 0 for the dense step
+    const int32_t *uniq;    // sparse step: the distinct ids (U of them, sc->n_unique)
+    int rsum_base;          // index of this launch's first per-CTA sum of r in rsum_part
 };
 
 __global__ void __launch_bounds__(kStateThreads)
@@ -606,38 +597,18 @@ k_state_dense(ColSource src, float *__restrict__ rsum_part, int nrsum, float *__
             }
             rsum = tsum;
         } else {
-            // sparse step: kRowBatch rows per thread at a time, their map
-            // entries and r loaded together; rows outside the batch's ids
-            // decay, touched rows add their sums of g^2
-            for (int64_t i0 = (int64_t)rb * kStateThreads + threadIdx.x; i0 < V; i0 += stride * kRowBatch) {
-                int sl[kRowBatch];
-                float rr[kRowBatch];
-#pragma unroll
-                for (int k = 0; k < kRowBatch; ++k) {
-                    const int64_t i = i0 + k * stride;
-                    sl[k] = (i < V) ? rowp.slot[i] : 0;
-                    rr[k] = (i < V) ? rowp.r[i] : 0.f;
-                }
-                float tsum = 0.f;
-#pragma unroll
-                for (int k = 0; k < kRowBatch; ++k) {
-                    const int64_t i = i0 + k * stride;
-                    if (i >= V)
-                        break;
-                    float mean_row = 0.f;
-                    if (sl[k]) {
-                        const int64_t u = sl[k] - 1;
-                        float tot = 0.f;
-                        for (int q = 0; q < rowp.nslices; ++q)
-                            tot += rowp.rowpart[u * rowp.nslices + q];
-                        mean_row = tot * inv_Df;
-                        rowp.slot[i] = 0;
-                    }
-                    const float rn = ema_pair(ema, rr[k], mean_row);
-                    rowp.r[i] = rn;
-                    tsum += rn;
-                }
-                rsum += tsum;
+            // sparse step: the touched rows only (the segment-sum kernel has
+            // decayed every other row): each adds its sums of g^2 per slice
+            const int64_t U = sc->n_unique;
+            for (int64_t u = (int64_t)rb * kStateThreads + threadIdx.x; u < U; u += stride) {
+                const int64_t i = rowp.uniq[u];
+                float tot = 0.f;
+                for (int q = 0; q < rowp.nslices; ++q)
+                    tot += rowp.rowpart[u * rowp.nslices + q];
+                const float rn = ema_pair(ema, rowp.r[i], tot * inv_Df);
+                rowp.r[i] = rn;
+                rowp.slot[i] = 0;
+                rsum += rn;
             }
         }
 #pragma unroll
@@ -650,7 +621,7 @@ k_state_dense(ColSource src, float *__restrict__ rsum_part, int nrsum, float *__
             float t = 0.f;
             for (int q = 0; q < kW; ++q)
                 t += part[q];
-            rsum_part[rb] = t;
+            rsum_part[rowp.rsum_base + rb] = t;
         }
     }
     if (threadIdx.x == 0) {
@@ -1266,7 +1237,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
         const ColSource src{nullptr, 0, sh.sums, sh.scales};
         e = launch_k(k_state_dense, dim3((D + kStateCols - 1) / kStateCols), dim3(kStateThreads), 0, a.stream,
                      false, src, rsum_part, 0, a.c, csum_part, sc, a.V, D, kc,
-                     RowPass{nullptr, nullptr, nullptr, 0, 0});
+                     RowPass{nullptr, nullptr, nullptr, 0, 0, nullptr, 0});
         if (e != cudaSuccess || ncta == 0)
             return e != cudaSuccess ? e : cudaGetLastError();
         const size_t cs_bytes = (size_t)D * sizeof(float);
@@ -1428,10 +1399,10 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
                          float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &kc,
                          cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
-                         int nslices, int nrow_ctas)
+                         int nslices, int nrow_ctas, const int32_t *uniq, int rsum_base)
 {
     const int ngroups = (D + kStateCols - 1) / kStateCols;
-    RowPass rp{r_rows, slot, rowpart, nslices, nrow_ctas};
+    RowPass rp{r_rows, slot, rowpart, nslices, nrow_ctas, uniq, rsum_base};
     const ColSource src{colpart, nparts, nullptr, nullptr};
     return launch_k(k_state_dense, dim3(ngroups + nrow_ctas), dim3(kStateThreads), 0, stream, pdl, src,
                     rsum_part, nrsum, c, csum_part, sc, V, D, kc, rp);

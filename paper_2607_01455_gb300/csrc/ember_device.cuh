@@ -135,6 +135,89 @@ __device__ __forceinline__ void store_w(void *W, int64_t idx, const float (&w)[V
     }
 }
 
+// L2 eviction-priority policies (createpolicy, fraction 1.0) and loads and
+// stores that carry one: evict_first for data touched for the last time in
+// a launch, so that it leaves L2 before data still to be reused.
+__device__ __forceinline__ uint64_t policy_evict_first()
+{
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last()
+{
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+
+template <int VEC>
+__device__ __forceinline__ typename Vec<VEC>::F load_g_hint(const float *p, uint64_t pol)
+{
+    if constexpr (VEC == 4) {
+        float4 v;
+        asm volatile("ld.global.nc.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                     : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                     : "l"(p), "l"(pol));
+        return v;
+    } else {
+        float v;
+        asm volatile("ld.global.nc.L2::cache_hint.f32 %0, [%1], %2;" : "=f"(v) : "l"(p), "l"(pol));
+        return v;
+    }
+}
+
+template <bool BF16, int VEC>
+__device__ __forceinline__ typename WRaw<BF16, VEC>::T load_w_hint(const void *W, int64_t idx, uint64_t pol)
+{
+    if constexpr (BF16 && VEC == 4) {
+        uint2 u;
+        asm volatile("ld.global.L2::cache_hint.v2.u32 {%0, %1}, [%2], %3;"
+                     : "=r"(u.x), "=r"(u.y)
+                     : "l"(static_cast<const unsigned short *>(W) + idx), "l"(pol));
+        return u;
+    } else if constexpr (!BF16 && VEC == 4) {
+        float4 v;
+        asm volatile("ld.global.L2::cache_hint.v4.f32 {%0, %1, %2, %3}, [%4], %5;"
+                     : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                     : "l"(static_cast<const float *>(W) + idx), "l"(pol));
+        return v;
+    } else {
+        return load_w<BF16, VEC>(W, idx);
+    }
+}
+
+template <bool BF16, int VEC>
+__device__ __forceinline__ void store_w_hint(void *W, int64_t idx, const float (&w)[VEC], uint64_t pol)
+{
+    if constexpr (BF16 && VEC == 4) {
+        const unsigned x = (unsigned)f2bf(w[0]) | ((unsigned)f2bf(w[1]) << 16);
+        const unsigned y = (unsigned)f2bf(w[2]) | ((unsigned)f2bf(w[3]) << 16);
+        asm volatile("st.global.L2::cache_hint.v2.u32 [%0], {%1, %2}, %3;" ::"l"(
+                         static_cast<unsigned short *>(W) + idx),
+                     "r"(x), "r"(y), "l"(pol)
+                     : "memory");
+    } else if constexpr (!BF16 && VEC == 4) {
+        asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(
+                         static_cast<float *>(W) + idx),
+                     "f"(w[0]), "f"(w[1]), "f"(w[2]), "f"(w[3]), "l"(pol)
+                     : "memory");
+    } else {
+        store_w<BF16, VEC>(W, idx, w);
+    }
+}
+
+template <int VEC>
+__device__ __forceinline__ void store_g_hint(float *p, const typename Vec<VEC>::F &v, uint64_t pol)
+{
+    if constexpr (VEC == 4)
+        asm volatile("st.global.L2::cache_hint.v4.f32 [%0], {%1, %2, %3, %4}, %5;" ::"l"(p), "f"(v.x), "f"(v.y),
+                     "f"(v.z), "f"(v.w), "l"(pol)
+                     : "memory");
+    else
+        asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(pol) : "memory");
+}
+
 __device__ __forceinline__ uint64_t now_ns()
 {
     uint64_t t;

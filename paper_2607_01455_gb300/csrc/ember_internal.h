@@ -218,6 +218,17 @@ struct StepConsts {
     EmaPair ema;
     float inv_D, inv_V, inv_bc;
 };
+// beta2 r + (1 - beta2) m in fp32 with the coefficients carried as float
+// pairs: within about an ulp of the fp64 value, and the fixed point stays
+// at r = m, which rounding beta2 and 1 - beta2 to single floats would shift
+// by about 1e-5 of r at beta2 = 0.999.  With m = 0 (a row outside a sparse
+// batch) it is the correctly rounded product beta2 r in all but near-tie
+// cases.
+__device__ __forceinline__ float ema_pair(const EmaPair &e, float r, float m)
+{
+    return fmaf(e.bh, r, fmaf(e.bl, r, fmaf(e.ah, m, e.al * m)));
+}
+
 inline StepConsts make_consts(double beta2, double one_minus_beta2, int64_t V, int64_t D, double inv_bc)
 {
     StepConsts k;
@@ -232,16 +243,19 @@ inline StepConsts make_consts(double beta2, double one_minus_beta2, int64_t V, i
 }
 
 // Column EMA and normaliser; with nrow_ctas > 0 the same launch also runs a
-// row pass: r for all V rows from per-slice sums of g^2, taken from
-// rowpart[slot[i]-1][nslices] for the sparse step (rows with slot 0 saw no
-// gradient) or, with slot == nullptr, from rowpart[nslices][V] for every row.
+// row pass: r from per-slice sums of g^2, taken from rowpart[u][nslices] for
+// the touched rows of the sparse step, or, with slot == nullptr, from
+// rowpart[nslices][V] for every row.
 // Column totals are exact fixed-point sums of the nparts partial rows
 // (ember_device.cuh); the normaliser's sum of r likewise over the nrsum
 // per-CTA sums in rsum_part.
+// For the sparse step (slot set) the row pass covers only the U touched rows
+// uniq[0..U) (the segment-sum kernel decays the others) and writes its
+// per-CTA sums of r from rsum_part[rsum_base] on.
 cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
                          float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &k,
                          cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
-                         int nslices, int nrow_ctas);
+                         int nslices, int nrow_ctas, const int32_t *uniq = nullptr, int rsum_base = 0);
 
 struct SparseArgs {
     int64_t V, D, N;

@@ -390,7 +390,9 @@ __global__ void __launch_bounds__(kThreads, kSparseCtasPerSm)
 k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             const int32_t *__restrict__ segidx, const DevScalars *__restrict__ sc,
             float *__restrict__ S, float *__restrict__ rowpart, float *__restrict__ carry,
-            float *__restrict__ colpart, int32_t *__restrict__ bounds, int D, int NS)
+            float *__restrict__ colpart, int32_t *__restrict__ bounds, int D, int NS,
+            float *__restrict__ r, const int32_t *__restrict__ slot, int64_t V, EmaPair ema,
+            float *__restrict__ rsum_part)
 {
     using F = typename Vec<VEC>::F;
     constexpr int R = 8;  // rows in flight per thread
@@ -415,6 +417,10 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
 #pragma unroll
     for (int e = 0; e < VEC; ++e)
         colacc[e] = 0.f;
+    // the occurrence rows stream through once: evict them first, so that
+    // the summed rows written here stay in L2 for the update that reads them
+    const uint64_t pol_rows = policy_evict_first();
+    const uint64_t pol_sums = policy_evict_last();
 
     const bool worker = w < nw && n_valid > 0;
     int p0 = 0, p1 = 0;
@@ -471,7 +477,7 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                 if (active) {
                     // an id seen once needs no summed row: the apply reads its occurrence row
                     if (len > 1)
-                        *reinterpret_cast<F *>(S + (int64_t)u * D + (int64_t)col * VEC) = acc;
+                        store_g_hint<VEC>(S + (int64_t)u * D + (int64_t)col * VEC, acc, pol_sums);
 #pragma unroll
                     for (int e = 0; e < VEC; ++e) {
                         const float a = comp(acc, e);
@@ -515,7 +521,7 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
                     if (p < we) {
                         uu[k] = sseg[p - wb];
                         if (active)
-                            v[k] = load_g<VEC>(rows + (int64_t)sperm[p - wb] * D + (int64_t)col * VEC);
+                            v[k] = load_g_hint<VEC>(rows + (int64_t)sperm[p - wb] * D + (int64_t)col * VEC, pol_rows);
                     }
                 }
 #pragma unroll
@@ -552,6 +558,46 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
 #pragma unroll
         for (int e = 0; e < VEC; ++e)
             out[col * VEC + e] = colacc[e];
+
+    // The rows outside the batch: r_i <- beta2 r_i (their g is 0), this CTA's
+    // share of the table, kRowBatch rows per thread at a time with their map
+    // entries loaded together; the touched rows are left to the state pass.
+    // The CTA's fp32 sum of the decayed r goes to rsum_part[blockIdx.x].
+    {
+        const int64_t i0 = (int64_t)blockIdx.x * V / gridDim.x, i1 = (int64_t)(blockIdx.x + 1) * V / gridDim.x;
+        float rsum = 0.f;
+        for (int64_t ib = i0 + threadIdx.x; ib < i1; ib += (int64_t)kThreads * kRowBatch) {
+            int sl[kRowBatch];
+            float rr[kRowBatch];
+#pragma unroll
+            for (int k = 0; k < kRowBatch; ++k) {
+                const int64_t i = ib + (int64_t)k * kThreads;
+                sl[k] = (i < i1) ? slot[i] : 1;
+                rr[k] = (i < i1) ? r[i] : 0.f;
+            }
+#pragma unroll
+            for (int k = 0; k < kRowBatch; ++k) {
+                if (sl[k] != 0)
+                    continue;
+                const float rn = ema_pair(ema, rr[k], 0.f);
+                r[ib + (int64_t)k * kThreads] = rn;
+                rsum += rn;
+            }
+        }
+        __shared__ float rsh[kThreads / 32];
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1)
+            rsum += __shfl_xor_sync(0xffffffffu, rsum, o);
+        if (lane == 0)
+            rsh[warp] = rsum;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float t = 0.f;
+            for (int q = 0; q < kThreads / 32; ++q)
+                t += rsh[q];
+            rsum_part[blockIdx.x] = t;
+        }
+    }
 }
 
 // Runs cut by worker boundaries.  CTA b handles boundary bd = b / NS + 1
@@ -685,6 +731,9 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
         cs[j] = (variant == EMBER_VARIANT_ROW) ? 1.f : sqrtf(c[j] * inv_bc * inv_s);
     __syncthreads();
 
+    // the summed rows, the W rows and the written W are touched for the last
+    // time in the step
+    const uint64_t pol = policy_evict_first();
     const int64_t stride = (int64_t)gridDim.x * rg * R;
     const int64_t ub0 = ((int64_t)blockIdx.x * rg + g) * R;
     // row ids (and, for ids seen once, the occurrence row) of the next
@@ -709,8 +758,8 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
             for (int cc = 0; cc < CPT; ++cc) {
                 const int col = l + cc * tpr;
                 if (row[k] >= 0 && col < DV) {
-                    gv[k][cc] = load_g<VEC>(src + (int64_t)col * VEC);
-                    wr[k][cc] = load_w<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC);
+                    gv[k][cc] = load_g_hint<VEC>(src + (int64_t)col * VEC, pol);
+                    wr[k][cc] = load_w_hint<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC, pol);
                 }
             }
         }
@@ -738,7 +787,7 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
                     const float u = comp(gv[k][cc], e) / den;
                     wv[e] = fmaf(lr_signed, u, wv[e]);
                 }
-                store_w<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC, wv);
+                store_w_hint<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC, wv, pol);
             }
         }
     }
@@ -857,18 +906,19 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     launch_sort_dedup(a, tr);
     const int G = kSparseCtas;
     const int nw = G / NS;
+    const StepConsts kc = make_consts(a.beta2, a.one_minus_beta2, a.V, a.D, a.inv_bc);
     launch_k(k_sp_segsum<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), a.rows, perm, segidx, sc, S,
-             rowpart, carry, colpart, bounds, D, NS);
+             rowpart, carry, colpart, bounds, D, NS, a.r, slot, a.V, kc.ema, rsum_part);
     tr.mark();
     launch_k(k_sp_carry<VEC>, dim3(G), dim3(kThreads), 0, a.stream, tr.pdl(), segidx, segoff, bounds, sc,
              carry, S, rowpart, colpart, D, NS, nw);
     tr.mark();
-    // row pass (all V rows) and column pass in one launch
-    const int64_t vb = (a.V + (int64_t)kStateThreads * kRowBatch - 1) / ((int64_t)kStateThreads * kRowBatch);
-    const int GV = (int)(vb < kGridCtas ? vb : kGridCtas);
-    const StepConsts kc = make_consts(a.beta2, a.one_minus_beta2, a.V, a.D, a.inv_bc);
-    launch_state(colpart, G, rsum_part, GV, a.c, csum_part, sc, a.V, D, kc, a.stream, tr.pdl(), a.r, slot, rowpart,
-                 NS, GV);
+    // the touched rows' r and the column pass in one launch; the per-CTA
+    // sums of r follow the segment-sum CTAs' sums of the decayed rows
+    const int64_t ub = (a.N + kStateThreads - 1) / kStateThreads;
+    const int GU = (int)(ub < kRsumParts - G ? ub : kRsumParts - G);
+    launch_state(colpart, G, rsum_part, G + GU, a.c, csum_part, sc, a.V, D, kc, a.stream, tr.pdl(), a.r, slot, rowpart,
+                 NS, GU, uniq, G);
     tr.mark();
     // one launch per column panel (one unless D is wider than a CTA's row)
     const int np = a.map.npanels, pw = a.map.pw;
