@@ -71,15 +71,17 @@ WORKLOADS = {
                  T=4096),
         # a quarter of the head's rows: the size the detailed profiles use
         Workload("lmhead_grad_v32768_d8192_t4096_bf16", 32768, 8192, "bf16", 20, kind="lmhead", T=4096),
+        Workload("dense_v32768_d8192_bf16", 32768, 8192, "bf16", 20, heavy_frac=0.01),
         # an LM head wider than one CTA's row (a 128256-token vocabulary at
         # hidden size 16384): the step runs in two column panels
         Workload("dense_wide_v128256_d16384_bf16", 128256, 16384, "bf16", 20, heavy_frac=0.01),
     ]
 }
-# The five workloads of the optimizer step in the order they are listed for
-# the paper's method; the LM-head gradient and wide-table workloads come
-# after them.
-ORDER = [n for n, w in WORKLOADS.items() if w.kind != "lmhead" and not n.startswith("dense_wide")]
+# The five workloads of the optimizer step, in the order they are listed for
+# the paper's method (the others are the LM-head gradient, the wide table and
+# the quarter-size tables the detailed profiles use).
+ORDER = ["dense_v1024_d64_f32", "dense_v32000_d4096_bf16", "dense_tied_v151936_d896_bf16",
+         "sparse_v262144_d2048_bf16_n32768", "dense_lmhead_v128256_d8192_bf16"]
 LOGIT_STD = 2.0
 
 
