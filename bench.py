@@ -4,10 +4,12 @@
 A step is one dense Ember step (row/column reduction, state update, apply)
 over one V x D table: by default the large LM head, V = 128256, D = 8192,
 bf16 weights, fp32 gradient and state.  Inputs are resident in HBM when the
-timed region starts; L2 is flushed (a 512 MiB write) between timed steps,
-outside the per-step CUDA events.  `value` is algorithmic bytes per step over
-the mean step time, summed over ranks (independent replicas: the step has no
-cross-GPU exchange on one table held whole by each GPU).  The same line
+timed region starts; L2 is flushed between timed steps, outside the per-step
+CUDA events: a 512 MiB write, then a 512 MiB read of another buffer, so that
+the step starts with a cold L2 that holds no dirty line of the flush.
+`value` is algorithmic bytes per step over the mean step time, summed over
+ranks (independent replicas: the step has no cross-GPU exchange on one table
+held whole by each GPU).  The same line
 carries one sub-object per workload of the method (`configs`: the 1024 x 64
 fp32 table, the 32000 x 4096 and 151936 x 896 bf16 tables, the sparse
 262144 x 2048 step with 32768 ids, and the LM head), each with its step
@@ -37,6 +39,24 @@ METRIC = "Ember step GB/s and % of GB300 HBM roofline (dense and sparse), params
 NOMINAL_HBM_GBS = 8000.0
 FALLBACK_HBM_GBS = 6800.0
 L2_FLUSH_BYTES = 512 << 20
+L2_NOTE = "flushed between steps (512 MiB write, then 512 MiB read; outside the events)"
+
+
+class L2Flush:
+    """Evicts L2 between timed steps: writes one buffer four times the size of
+    L2, then reads another of the same size, so that the write's dirty lines
+    are written back here and not inside the next step."""
+
+    def __init__(self, dev):
+        import torch
+        self.w = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+        self.r = torch.ones(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+        self.out = torch.empty((), dtype=torch.float32, device=dev)
+
+    def __call__(self):
+        import torch
+        self.w.zero_()
+        torch.amax(self.r, dim=0, out=self.out)
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) per launch of a
 # dominant kernel, from an ncu capture of the kernel as it is now, with where
@@ -135,7 +155,7 @@ def run_dense(wl, dev, steps, warmup, flush, seed=0, clocks_for=None):
     warm_ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
     for i in range(warmup):
         t += 1
-        flush.zero_()
+        flush()
         emb.trace(warm_ev if (three and i % 2) else [])
         emb.step_dense(W, G, wl.lr, t)
     torch.cuda.synchronize()
@@ -149,7 +169,7 @@ def run_dense(wl, dev, steps, warmup, flush, seed=0, clocks_for=None):
     with sampler:
         for k in range(steps):
             t += 1
-            flush.zero_()
+            flush()
             emb.trace(kern_ev.get(k, []))
             step_ev[k][0].record(stream)
             emb.step_dense(W, G, wl.lr, t)
@@ -222,7 +242,7 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
     warm = [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)]
     for i in range(warmup):
         t += 1
-        flush.zero_()
+        flush()
         emb.trace(warm if i % 2 else [])
         emb.step_sparse(W, ids, rows, wl.lr, t)
     torch.cuda.synchronize()
@@ -234,7 +254,7 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
     kern_ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for k in traced}
     for k in range(steps):
         t += 1
-        flush.zero_()
+        flush()
         emb.trace(kern_ev.get(k, []))
         step_ev[k][0].record()
         emb.step_sparse(W, ids, rows, wl.lr, t)
@@ -256,7 +276,7 @@ def run_sparse(wl, dev, steps, warmup, flush, seed=0):
         emb.step_sparse(W, ids, rows, wl.lr, t + 1, stream=side)
     gev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     for k in range(steps):
-        flush.zero_()
+        flush()
         gev[k][0].record()
         graph.replay()
         gev[k][1].record()
@@ -284,12 +304,12 @@ def run_row_only(wl, dev, steps, warmup, flush, W, G):
     t = 0
     for _ in range(warmup):
         t += 1
-        flush.zero_()
+        flush()
         emb.step_dense(W, G, wl.lr, t)
     ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
     for k in range(steps):
         t += 1
-        flush.zero_()
+        flush()
         ev[k][0].record()
         emb.step_dense(W, G, wl.lr, t)
         ev[k][1].record()
@@ -327,7 +347,7 @@ def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
     t = 0
     for _ in range(warmup):
         t += 1
-        flush.zero_()
+        flush()
         emb.step_lmhead(W, dl, h, G, wl.lr, t)
     torch.cuda.synchronize()
     step_ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
@@ -336,7 +356,7 @@ def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
     kern_ev = {k: [torch.cuda.Event(enable_timing=True) for _ in range(nk + 1)] for k in traced}
     for k in range(steps):
         t += 1
-        flush.zero_()
+        flush()
         emb.trace(kern_ev.get(k, []))
         step_ev[k][0].record()
         emb.step_lmhead(W, dl, h, G, wl.lr, t)
@@ -362,13 +382,13 @@ def run_lmhead(wl, dev, steps, warmup, flush, seed=0):
         cublas_out = "bf16 then converted"
     for _ in range(warmup):
         t += 1
-        flush.zero_()
+        flush()
         emb2.step_dense(W, gemm(), wl.lr, t)
     torch.cuda.synchronize()
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(steps)]
     for k in range(steps):
         t += 1
-        flush.zero_()
+        flush()
         ev[k][0].record()
         Gc = gemm()
         ev[k][1].record()
@@ -580,7 +600,7 @@ def sparse_kernel_bytes(wl, U):
 
 def run_sparse_line(args, wl, world, rank, dev):
     import torch
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush = L2Flush(dev)
     barrier(world)
     with ClockSampler(dev.index or 0) as clocks:
         sp = run_sparse(wl, dev, args.steps, args.warmup, flush, seed=rank)
@@ -592,7 +612,7 @@ def run_sparse_line(args, wl, world, rank, dev):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic",
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "N": wl.N, "w_dtype": wl.wdtype,
-                   "ids": "int64", "l2": "flushed between steps (512 MiB write, outside the events)",
+                   "ids": "int64", "l2": L2_NOTE,
                    "parallelism": f"replicas x{world}"},
         "roofline": sp["roofline"],
         "cpu_baseline": None, "e2e": None, "gpu_launches": sp["gpu_launches"],
@@ -608,7 +628,7 @@ def run_lmhead_line(args, wl, world, rank, dev):
     (ember_step_lmhead) is the step; value = its HBM bytes per second (G
     written and read once, W read and written, dlogits and H read)."""
     import torch
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush = L2Flush(dev)
     barrier(world)
     with ClockSampler(dev.index or 0) as clocks:
         lm = run_lmhead(wl, dev, args.steps, args.warmup, flush, seed=rank)
@@ -620,7 +640,7 @@ def run_lmhead_line(args, wl, world, rank, dev):
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16 x bf16 -> f32",
         "data": "synthetic",
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "T": wl.T, "w_dtype": wl.wdtype,
-                   "l2": "inputs larger than L2, and flushed between steps (512 MiB write, outside the events)",
+                   "l2": "inputs larger than L2, and " + L2_NOTE,
                    "parallelism": f"replicas x{world}"},
         "roofline": lm["roofline"], "cpu_baseline": None, "e2e": None, "gpu_launches": lm["gpu_launches"],
         "clocks": clocks.summary(), "lmhead_fused": lm,
@@ -652,7 +672,7 @@ def run_ours(args, world, rank, local):
     if wl.kind == "sparse":
         return run_sparse_line(args, wl, world, rank, dev)
 
-    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+    flush = L2Flush(dev)
     peak, peak_kind = measured_hbm_peak()
     # clocks sampled over every timed region of the run (the main step first)
     with ClockSampler(local) as clocks:
@@ -696,7 +716,7 @@ def run_ours(args, world, rank, local):
             ts = []
             for _ in range(n_e2e):
                 t += 1
-                flush.zero_()
+                flush()
                 e0.record(stream)
                 G2.copy_(Gh, non_blocking=True)
                 emb.step_dense(W, G2, wl.lr, t)
@@ -710,7 +730,7 @@ def run_ours(args, world, rank, local):
             ts = []
             for _ in range(n_e2e):
                 t += 1
-                flush.zero_()
+                flush()
                 e0.record(stream)
                 emb.step_dense_from_host(W, Gh, G2, wl.lr, t)
                 Sh.copy_(emb.state, non_blocking=True)
@@ -771,7 +791,7 @@ def run_ours(args, world, rank, local):
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f32", "data": "synthetic",
         "config": {"workload": wl.name, "V": wl.V, "D": wl.D, "w_dtype": wl.wdtype, "g_dtype": "f32",
-                   "state_dtype": "f32", "l2": "flushed between steps (512 MiB write, outside the events)",
+                   "state_dtype": "f32", "l2": L2_NOTE,
                    "parallelism": f"replicas x{world}"},
         "roofline": main["roofline"],
         "cpu_baseline": cpu,

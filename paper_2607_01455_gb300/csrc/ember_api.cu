@@ -574,12 +574,6 @@ ember_status ember_get_device_status(ember_handle *h, void *stream)
     if (flags && (cudaMemsetAsync(&sc->flags, 0, sizeof(unsigned), s) != cudaSuccess ||
                   cudaStreamSynchronize(s) != cudaSuccess))
         return EMBER_ERR_CUDA;
-    // a wait that gave up leaves the grid-barrier words of the one-launch
-    // steps set (abort, partial arrivals): clear them so the next step runs
-    if ((flags & kFlagTimeout) &&
-        (cudaMemsetAsync(&sc->bar_count, 0, 4 * sizeof(unsigned), s) != cudaSuccess ||
-         cudaStreamSynchronize(s) != cudaSuccess))
-        return EMBER_ERR_CUDA;
     if (flags & kFlagTimeout)
         return EMBER_ERR_TIMEOUT;
     if (flags & kFlagIdRange)

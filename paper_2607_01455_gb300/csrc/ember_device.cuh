@@ -232,58 +232,6 @@ __device__ __forceinline__ unsigned ld_acquire(const unsigned *p)
     return v;
 }
 
-// Grid-wide barrier for a cooperative launch (every CTA co-resident), with a
-// bounded wait.  count: arrivals at the current barrier (returned to zero
-// by the last arriver); gen: barriers completed; abort: set by a CTA whose
-// wait ran past limit_ns, after which this and every later barrier fails at
-// once.  A CTA that sees false must return without touching shared results.
-// The pattern of the CUDA programming model's grid synchronisation: the CTA
-// barrier orders the CTA's writes before thread 0's fence and arrival; the
-// waiters' acquire loads order everything after it.  *t_release (optional)
-// receives the release time from the last arriver.
-static __device__ __noinline__ bool grid_sync(unsigned *count, unsigned *gen, unsigned *abort, unsigned *flags,
-                                       unsigned timeout_bit, unsigned nblocks, uint64_t limit_ns,
-                                       unsigned long long *t_release)
-{
-    __shared__ int ok_sh;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        int ok = 1;
-        const unsigned g0 = ld_acquire(gen);
-        __threadfence();
-        const unsigned arrived = atomicAdd(count, 1u) + 1u;
-        if (arrived == nblocks) {
-            atomicExch(count, 0u);
-            if (t_release)
-                *t_release = now_ns();
-            __threadfence();
-            atomicAdd(gen, 1u);
-        } else {
-            const uint64_t t0 = now_ns();
-            for (unsigned k = 1; ld_acquire(gen) == g0; ++k) {
-                if ((k & 15u) == 0) {
-                    if (ld_acquire(abort)) {
-                        ok = 0;
-                        break;
-                    }
-                    if (now_ns() - t0 > limit_ns) {
-                        atomicOr(flags, timeout_bit);
-                        atomicExch(abort, 1u);
-                        ok = 0;
-                        break;
-                    }
-                }
-            }
-        }
-        if (ok && ld_acquire(abort))
-            ok = 0;
-        __threadfence();
-        ok_sh = ok;
-    }
-    __syncthreads();
-    return ok_sh != 0;
-}
-
 // ---------------------------------------------------------------------------
 // Exact sums of non-negative fp32 values in 64-bit fixed point.
 //

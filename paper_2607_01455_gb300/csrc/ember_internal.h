@@ -50,11 +50,6 @@ struct DevScalars {
     unsigned flags;    // sticky device error bits (kFlag*)
     int32_t n_unique;  // sparse step: number of distinct valid ids
     int32_t n_valid;   // sparse step: number of ids inside [0, V)
-    // grid barrier of kernels whose CTAs wait on one another (cooperative
-    // launches): arrivals at the current barrier, barriers completed, and a
-    // word set when a bounded wait gave up (every later barrier then fails
-    // at once until ember_get_device_status clears it)
-    unsigned bar_count, bar_gen, bar_abort, bar_pad;
 };
 
 // Sparse step: ids are sorted in tiles of kSortTile keys by kSortThreads

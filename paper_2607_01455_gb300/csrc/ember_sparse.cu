@@ -409,6 +409,8 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
     const int nw = gridDim.x / NS;
     const int col = sigma * kThreads + threadIdx.x;
     const bool active = col < DV;
+    // threads past the row's end load its last vector (and discard the sums)
+    const float *src = rows + (int64_t)(active ? col : DV - 1) * VEC;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     grid_dep_wait();  // runs and occurrence order from the dedup kernels
     grid_dep_launch();
@@ -511,28 +513,29 @@ k_sp_segsum(const float *__restrict__ rows, const int32_t *__restrict__ perm,
             }
             __syncthreads();
             for (int pb = wb; pb < we; pb += R) {
+                // R rows in flight; only the window's last batch is partial
+                const int nb = (we - pb < R) ? we - pb : R;
+                const int *bp = sperm + (pb - wb);
                 F v[R];
-                int uu[R];
+                if (nb == R) {
 #pragma unroll
-                for (int k = 0; k < R; ++k) {
-                    const int p = pb + k;
-                    uu[k] = -1;
-                    v[k] = zero_vec<VEC>();
-                    if (p < we) {
-                        uu[k] = sseg[p - wb];
-                        if (active)
-                            v[k] = load_g_hint<VEC>(rows + (int64_t)sperm[p - wb] * D + (int64_t)col * VEC, pol_rows);
-                    }
+                    for (int k = 0; k < R; ++k)
+                        v[k] = load_g_hint<VEC>(src + (int64_t)bp[k] * D, pol_rows);
+                } else {
+#pragma unroll
+                    for (int k = 0; k < R; ++k)
+                        v[k] = (k < nb) ? load_g_hint<VEC>(src + (int64_t)bp[k] * D, pol_rows) : zero_vec<VEC>();
                 }
 #pragma unroll
                 for (int k = 0; k < R; ++k) {
-                    if (uu[k] < 0)
+                    if (k >= nb)
                         break;
-                    if (uu[k] != cur) {
+                    const int u = sseg[pb - wb + k];
+                    if (u != cur) {
                         flush(cur);
                         acc = zero_vec<VEC>();
                         cmp = zero_vec<VEC>();
-                        cur = uu[k];
+                        cur = u;
                         len = 0;
                     }
                     ++len;

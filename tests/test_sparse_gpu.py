@@ -89,6 +89,10 @@ def test_dedup_bit_exact(cuda_device, V, D, N, idtype):
 @pytest.mark.parametrize("V,D,N", [
     (64, 4, 100), (1000, 64, 512), (1000, 203, 3000), (4096, 256, 8192),
     (30000, 896, 6000), (2000, 2048, 5000),
+    # two column slices of the segment sums, the second 8 columns wide
+    # (1032 = 1024 + 8), and bf16 rows that do not start on 16-byte
+    # boundaries (1100 = 8 * 137 + 4)
+    (1500, 1032, 2500), (3000, 1100, 4000),
 ])
 @pytest.mark.parametrize("wdtype", ["bf16", "f32"])
 def test_sparse_parity(cuda_device, V, D, N, wdtype):
