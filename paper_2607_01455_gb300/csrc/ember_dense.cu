@@ -313,7 +313,7 @@ __device__ __forceinline__ void apply_rows(void *__restrict__ W, const float *__
 #pragma unroll
                 for (int e = 0; e < VEC; ++e) {
                     const float den = fmaf(rs, cs[col * VEC + e], eps);
-                    const float u = comp(gv[k][cc], e) / den;
+                    const float u = update_ratio(comp(gv[k][cc], e), den);
                     w[e] = fmaf(lr_signed, u, w[e]);
                 }
                 store_w<BF16, VEC>(W, (i - span.row_base) * ld + (int64_t)col * VEC, w);
@@ -907,7 +907,7 @@ k_dense_cluster(SmallArgs a)
 #pragma unroll
                 for (int e = 0; e < VEC; ++e) {
                     const float den = fmaf(rs, cs[col * VEC + e], a.eps);
-                    const float u = comp(gv, e) / den;
+                    const float u = update_ratio(comp(gv, e), den);
                     wv[e] = fmaf(a.lr_signed, u, wv[e]);
                 }
                 store_w<BF16, VEC>(a.W, i * D + (int64_t)col * VEC, wv);
@@ -1095,7 +1095,7 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
                 unpack_w(wr[k][c], w);
 #pragma unroll
                 for (int e = 0; e < VEC; ++e)
-                    w[e] = fmaf(lr_signed, comp(v[k][c], e) / den, w[e]);
+                    w[e] = fmaf(lr_signed, update_ratio(comp(v[k][c], e), den), w[e]);
                 store_w<BF16, VEC>(W, i * D + (int64_t)col * VEC, w);
             }
         }

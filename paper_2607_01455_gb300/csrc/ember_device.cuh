@@ -218,6 +218,13 @@ __device__ __forceinline__ void store_g_hint(float *p, const typename Vec<VEC>::
         asm volatile("st.global.L2::cache_hint.f32 [%0], %1, %2;" ::"l"(p), "f"(v), "l"(pol) : "memory");
 }
 
+// The update ratio g / (sqrt(rhat_i) sqrt(chat_j / s) + eps) of Algorithm 1,
+// with the fast reciprocal-and-multiply division (within 2 fp32 ulps for a
+// denominator below 2^126; the denominator here is a gradient-sized positive
+// number).  Every kernel that applies an update uses this one form, so the
+// dense, sparse, one-launch and sharded steps stay bitwise identical.
+__device__ __forceinline__ float update_ratio(float g, float den) { return __fdividef(g, den); }
+
 __device__ __forceinline__ uint64_t now_ns()
 {
     uint64_t t;

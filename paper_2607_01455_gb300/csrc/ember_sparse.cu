@@ -787,7 +787,7 @@ k_sp_apply(void *__restrict__ W, const float *__restrict__ S, const float *__res
 #pragma unroll
                 for (int e = 0; e < VEC; ++e) {
                     const float den = fmaf(rs, cs[col * VEC + e], eps);
-                    const float u = comp(gv[k][cc], e) / den;
+                    const float u = update_ratio(comp(gv[k][cc], e), den);
                     wv[e] = fmaf(lr_signed, u, wv[e]);
                 }
                 store_w_hint<BF16, VEC>(W, row[k] * ld + (int64_t)col * VEC, wv, pol);
