@@ -105,7 +105,7 @@ def sparse_bytes(wl, U):
     return 4 * N * D + 8 * N + min(8 * U * D, 4 * N * D) + 2 * w * U * D + 8 * V + 8 * D
 
 
-SPARSE_KERNELS = ("tile_sort", "rank", "scatter", "heads", "segments", "segsum", "carry",
+SPARSE_KERNELS = ("tile_sort", "rank", "scatter", "segments", "segsum", "carry",
                   "rows_and_state", "apply")
 TRACE_EVERY = 4  # every 4th timed step records kernel-boundary events
 

@@ -17,10 +17,14 @@
 //             floating-point data: 1024-key tiles are bitonic-sorted in shared
 //             memory, then every key's global rank is its rank in its tile
 //             plus its lower bound in every other tile (integer atomics, so
-//             the rank is exact and the order deterministic).
-//   dedup     k_sp_heads, k_sp_segments: run heads, the distinct ids
-//             (ascending), where each id's run starts, and a V-entry map from
-//             a touched row to its distinct-id index.
+//             the rank is exact and the order deterministic).  The same
+//             searches find the run heads: a key heads its id's run unless
+//             some tile holds a smaller key of the same id, which is then the
+//             key just below it in that tile.  The scatter counts the heads
+//             and the valid ids of every tile of sorted positions.
+//   dedup     k_sp_segments: the distinct ids (ascending), where each id's
+//             run starts, and a V-entry map from a touched row to its
+//             distinct-id index.
 //   segsum    k_sp_segsum, k_sp_carry: the summed gradient row of every
 //             distinct id, adding its occurrences in increasing occurrence
 //             order (compensated fp32 sums); per (id, column slice) sums of
@@ -50,6 +54,9 @@ namespace {
 using namespace dev;
 
 constexpr uint64_t kPad = ~0ull;
+// Bit of a key's rank word set when the key is not the head of its id's run
+// (ranks stay below 2^30: N <= INT32_MAX / 2).
+constexpr int kNotHead = 1 << 30;
 constexpr int kKeysPerThread = kSortTile / kSortThreads;
 
 // keys a <= b afterwards when `up`, a >= b otherwise
@@ -78,7 +85,7 @@ __device__ __forceinline__ uint64_t shfl_xor_u64(uint64_t x, int m)
 template <typename IdT>
 __global__ void __launch_bounds__(kSortThreads)
 k_sp_tile_sort(const IdT *__restrict__ ids, int64_t N, int64_t V, uint64_t *__restrict__ keys,
-               int32_t *__restrict__ rank, DevScalars *sc)
+               int32_t *__restrict__ rank, int32_t *__restrict__ tilecnt, DevScalars *sc)
 {
     static_assert(kSortTile == 4 * kSortThreads, "four keys per thread");
     __shared__ uint64_t s[kSortTile];
@@ -139,15 +146,27 @@ k_sp_tile_sort(const IdT *__restrict__ ids, int64_t N, int64_t V, uint64_t *__re
             }
         }
     }
+    // rank within the tile, and kNotHead where the key before it in the
+    // tile has the same id; the scatter's counts of this tile start at zero
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+        s[4 * t + q] = key[q];
+    if (t < 2)
+        tilecnt[2 * blockIdx.x + t] = 0;
+    __syncthreads();
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-        keys[base + 4 * t + q] = key[q];
-        rank[base + 4 * t + q] = 4 * t + q;
+        const int i = 4 * t + q;
+        const bool same = i > 0 && (s[i - 1] >> 32) == (key[q] >> 32);
+        keys[base + i] = key[q];
+        rank[base + i] = i | (same ? kNotHead : 0);
     }
 }
 
 // CTA (own, other): add to each key of tile `own` the number of keys of tile
-// `other` below it.  Keys are unique, so the ranks form a permutation.
+// `other` below it.  Keys are unique, so the ranks form a permutation.  A key
+// whose lower bound in `other` follows a key of the same id is not the head
+// of its id's run.
 __global__ void __launch_bounds__(kSortThreads)
 k_sp_rank(const uint64_t *__restrict__ keys, int32_t *__restrict__ rank)
 {
@@ -177,21 +196,44 @@ k_sp_rank(const uint64_t *__restrict__ keys, int32_t *__restrict__ rank)
             else
                 hi = mid;
         }
-        if (lo)
+        if (lo) {
             atomicAdd(&rank[at], lo);
+            if ((s[lo - 1] >> 32) == (x >> 32))
+                atomicOr(&rank[at], kNotHead);
+        }
     }
 }
 
+// Keys to their sorted positions, and per tile of sorted positions the
+// number of run heads and of valid ids (counted per warp, then one integer
+// atomic per tile a warp touches).  npad is a multiple of the warp size, so
+// every lane of a warp takes the same iterations.
 __global__ void k_sp_scatter(const uint64_t *__restrict__ keys, const int32_t *__restrict__ rank,
-                             int64_t npad, uint64_t *__restrict__ sorted)
+                             int64_t npad, int64_t V, uint64_t *__restrict__ sorted, int32_t *__restrict__ tilecnt)
 {
     grid_dep_wait();  // ranks
     grid_dep_launch();
+    const int lane = threadIdx.x & 31;
     for (int64_t q = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; q < npad;
          q += (int64_t)gridDim.x * blockDim.x) {
         const uint64_t x = keys[q];
-        if (x != kPad)
-            sorted[rank[q]] = x;
+        const int rk = rank[q];
+        const bool real = x != kPad;
+        const int pos = rk & ~kNotHead;
+        if (real)
+            sorted[pos] = x;
+        const bool valid = real && (int64_t)(x >> 32) < V;
+        const bool head = valid && !(rk & kNotHead);
+        const int tile = real ? pos / kSortTile : -1;
+        const unsigned peers = __match_any_sync(0xffffffffu, tile);
+        const int nh = __popc(__ballot_sync(0xffffffffu, head) & peers);
+        const int nv = __popc(__ballot_sync(0xffffffffu, valid) & peers);
+        if (real && lane == __ffs(peers) - 1) {
+            if (nh)
+                atomicAdd(&tilecnt[2 * tile], nh);
+            if (nv)
+                atomicAdd(&tilecnt[2 * tile + 1], nv);
+        }
     }
 }
 
@@ -209,34 +251,6 @@ __device__ __forceinline__ int block_sum_int(int x, int *sh)
         t += sh[q];
     __syncthreads();
     return t;
-}
-
-// Per tile of the sorted keys: number of run heads and of valid ids.
-__global__ void __launch_bounds__(kSortThreads)
-k_sp_heads(const uint64_t *__restrict__ sorted, int64_t N, int64_t V, int32_t *__restrict__ tilecnt)
-{
-    __shared__ int sh[kSortThreads / 32];
-    grid_dep_wait();  // sorted keys
-    grid_dep_launch();
-    const int64_t p0 = (int64_t)blockIdx.x * kSortTile + (int64_t)threadIdx.x * kKeysPerThread;
-    int nh = 0, nv = 0;
-#pragma unroll
-    for (int q = 0; q < kKeysPerThread; ++q) {
-        const int64_t p = p0 + q;
-        if (p < N) {
-            const uint64_t id = sorted[p] >> 32;
-            if ((int64_t)id < V) {
-                ++nv;
-                nh += (p == 0 || (sorted[p - 1] >> 32) != id);
-            }
-        }
-    }
-    nh = block_sum_int(nh, sh);
-    nv = block_sum_int(nv, sh);
-    if (threadIdx.x == 0) {
-        tilecnt[2 * blockIdx.x] = nh;
-        tilecnt[2 * blockIdx.x + 1] = nv;
-    }
 }
 
 // Distinct ids and their runs.  Thread t of tile b owns sorted positions
@@ -838,19 +852,18 @@ void launch_sort_dedup(const SparseArgs &a, Tracer &tr)
         const int64_t npad = (int64_t)T * kSortTile;
         if (a.ids64)
             launch_k(k_sp_tile_sort<int64_t>, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(),
-                     static_cast<const int64_t *>(a.ids), a.N, a.V, keys, rank, sc);
+                     static_cast<const int64_t *>(a.ids), a.N, a.V, keys, rank, tilecnt, sc);
         else
             launch_k(k_sp_tile_sort<int32_t>, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(),
-                     static_cast<const int32_t *>(a.ids), a.N, a.V, keys, rank, sc);
+                     static_cast<const int32_t *>(a.ids), a.N, a.V, keys, rank, tilecnt, sc);
         tr.mark();
         if (T > 1) {
             launch_k(k_sp_rank, dim3(T, T), dim3(kSortThreads), 0, a.stream, tr.pdl(), keys, rank);
             tr.mark();
         }
         const int nsc = (int)((npad + kThreads - 1) / kThreads);
-        launch_k(k_sp_scatter, dim3(nsc), dim3(kThreads), 0, a.stream, tr.pdl(), keys, rank, npad, sorted);
-        tr.mark();
-        launch_k(k_sp_heads, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V, tilecnt);
+        launch_k(k_sp_scatter, dim3(nsc), dim3(kThreads), 0, a.stream, tr.pdl(), keys, rank, npad, a.V, sorted,
+                 tilecnt);
         tr.mark();
         launch_k(k_sp_segments, dim3(T), dim3(kSortThreads), 0, a.stream, tr.pdl(), sorted, a.N, a.V,
                  tilecnt, uniq, segoff, perm, segidx, slot, single, sc);
