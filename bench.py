@@ -63,15 +63,16 @@ class L2Flush:
 # it came from.  A kernel that changes gets None here until it is captured
 # again.
 TRAFFIC = {
-    # the 32768 x 8192 quarter table measured 2.1166 GB per launch (mean of
+    # the 32768 x 8192 quarter table measured 2.1156 GB per launch (mean of
     # two launches); every row of G and W is read once and W written once,
     # so the traffic is scaled by rows
     ("k_apply_dense", "dense_lmhead_v128256_d8192_bf16"): (
-        int(2.1166e9 * 128256 / 32768),
+        int(2.1156e9 * 128256 / 32768),
         "ncu dram__bytes_read.sum + dram__bytes_write.sum of k_apply_dense on the 32768 x 8192 table, "
-        "2.1166 GB per launch, scaled by rows (2026-12-02)"),
+        "2.1156 GB per launch, scaled by rows (2026-12-02, reciprocal-multiply division)"),
     ("k_sp_segsum", "sparse_v262144_d2048_bf16_n32768"): (
-        274110720, "ncu dram__bytes_read.sum + dram__bytes_write.sum of k_sp_segsum on this workload (2026-12-02)"),
+        274328064, "ncu dram__bytes_read.sum + dram__bytes_write.sum of k_sp_segsum on this workload "
+                   "(2026-12-02, full-batch loop)"),
     # k_lmhead_grad: the re-reads of its operands do not grow in proportion
     # to the rows (3.2 x the algorithmic reads at 32768 rows), so no
     # full-size figure is derived from the quarter-size capture

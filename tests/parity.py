@@ -16,12 +16,13 @@ floor therefore also takes the oracle's own step |W_t - W_{t-1}| when the
 previous weights are given.
 
 One refinement of the bf16 bar, derived from the arithmetic: the kernel
-forms W - lr u in fp32 (the paper fixes no precision), so the new weight
-carries an error of a few fp32 ulps of the step |W_t - W_{t-1}| (about
-4 * 2^-24 of it).  Rounding to bf16 can then land more than one bf16 ulp
+forms W - lr u in fp32 (the paper fixes no precision), with u from a
+reciprocal and a multiply (within 2 fp32 ulps), so the new weight carries an
+error of a few fp32 ulps of the step |W_t - W_{t-1}| (at most about
+8 * 2^-24 of it).  Rounding to bf16 can then land more than one bf16 ulp
 (2^-8 of |W_t|) away from the oracle's rounding only where that error
 exceeds a bf16 ulp of the result, i.e. where the step nearly cancels the
-weight: |W_t| < 2^-14 |W_t - W_{t-1}|.  Every element more than 1 ulp apart
+weight: |W_t| < 2^-13 |W_t - W_{t-1}|.  Every element more than 1 ulp apart
 must lie in that set (with a margin: |W_t| <= 2^-12 of the step, or of lr
 when the previous weights are not given) and meet the fp32-weight bar
 |got - want| <= 1e-5 max(|want|, lr, step).  There is no count cap: the
