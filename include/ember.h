@@ -164,7 +164,7 @@ ember_status ember_bind_workspace(ember_handle *h, void *workspace, size_t bytes
  * scalar path gives the same results more slowly.
  *   A small table (V * D <= 65536 on the vector path, whose rows a CTA
  * covers in a few passes) runs as one launch of a thread-block cluster of
- * up to 8 CTAs that keeps G and W in shared memory and reads G from HBM
+ * up to 16 CTAs that keeps G and W in shared memory and reads G from HBM
  * once; every other table runs as three launches (reduce, column
  * statistics and normaliser, update), chained with programmatic dependent
  * launch.  Both forms run the same arithmetic on the same CTA row

@@ -79,6 +79,31 @@ using namespace dev;
 // and colpart: a column panel of a wider table has D < ld, and then each
 // row's sum of g^2 over the panel goes to rowpart[i] instead of into r.
 // ---------------------------------------------------------------------------
+// Column partial of a CTA from its row groups' sums: every group's sums side
+// by side in rg x D floats of shared memory, then each column added over
+// the groups in order 0 .. rg-1 -- the same float sums as a running total
+// over the groups, with one barrier instead of one per group.
+template <int VEC, int CPT>
+__device__ __forceinline__ void combine_row_groups(const float (&acc)[CPT][VEC], float *colsh, float *out, int D,
+                                                   int DV, int tpr, int rg, int g, int l)
+{
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) {
+        const int col = l + c * tpr;
+        if (col < DV)
+#pragma unroll
+            for (int e = 0; e < VEC; ++e)
+                colsh[(size_t)g * D + col * VEC + e] = acc[c][e];
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < D; j += kThreads) {
+        float t = colsh[j];
+        for (int q = 1; q < rg; ++q)
+            t += colsh[(size_t)q * D + j];
+        out[j] = t;
+    }
+}
+
 template <int VEC, int CPT, int R, bool STAGE, bool KEEP = false>
 __device__ __forceinline__ void reduce_rows(const float *__restrict__ G, float *__restrict__ r,
                                             float *__restrict__ colpart_row, float *__restrict__ rsum_out,
@@ -214,22 +239,7 @@ __device__ __forceinline__ void reduce_rows(const float *__restrict__ G, float *
                     colpart_row[col * VEC + e] = acc[c][e];
         }
     } else {
-        float *colsh = comb;  // D floats of shared memory
-        for (int q = 0; q < rg; ++q) {
-            if (g == q) {
-#pragma unroll
-                for (int c = 0; c < CPT; ++c) {
-                    const int col = l + c * tpr;
-                    if (col < DV)
-#pragma unroll
-                        for (int e = 0; e < VEC; ++e)
-                            colsh[col * VEC + e] = (q == 0) ? acc[c][e] : colsh[col * VEC + e] + acc[c][e];
-                }
-            }
-            __syncthreads();
-        }
-        for (int j = tid; j < D; j += kThreads)
-            colpart_row[j] = colsh[j];
+        combine_row_groups<VEC, CPT>(acc, comb, colpart_row, D, DV, tpr, rg, g, l);  // rg x D floats
     }
 
     // sum of the new r values of this CTA (fp32): fixed butterfly per warp,
@@ -532,7 +542,7 @@ k_reduce_dense(const float *__restrict__ G, float *__restrict__ r, float *__rest
 {
     grid_dep_wait();    // the first kernel of a step: returns at once
     grid_dep_launch();  // the state pass may start launching now; it waits for this grid
-    extern __shared__ float comb_sh[];  // D floats: the row groups' column sums combined
+    extern __shared__ float comb_sh[];  // rg x D floats: the row groups' column sums
     reduce_rows<VEC, CPT, R, STAGE>(G, r, colpart + (int64_t)blockIdx.x * ld, rsum_part + blockIdx.x, V, D, ld,
                                     tpr, kc, G_stage, rowpart, span, blockIdx.x, comb_sh,
                                     nullptr);
@@ -686,7 +696,7 @@ k_apply_dense(void *__restrict__ W, const float *__restrict__ G, const float *__
 }
 
 // ---------------------------------------------------------------------------
-// Small tables in one launch: one thread-block cluster of nparts <= 8 CTAs
+// Small tables in one launch: one thread-block cluster of nparts <= 16 CTAs
 // (the same CTA grid and row ranges as the three-launch form).  Each CTA
 //   - starts copying its rows of W into shared memory (cp.async) and loads
 //     the old c;
@@ -735,8 +745,9 @@ struct SmallArgs {
 
 // Shared memory of k_dense_cluster, from the dynamic base: kept G, kept W
 // (one 16- or 8-byte slot per thread, per row and access of each reduce
-// iteration), then D floats each of the column partial, the combine buffer,
-// the old c, the new c (then the column scales), and ceil(D/32) floats.
+// iteration), then D floats of the column partial, (256 / tpr) x D floats of
+// the row groups' sums, D floats each of the old c and the new c (then the
+// column scales), and ceil(D/32) floats.
 template <int CPT, int R, bool BF16>
 __host__ __device__ constexpr size_t small_slots(int nits) { return (size_t)nits * R * CPT * kThreads; }
 
@@ -751,12 +762,15 @@ bool small_table_plan(int64_t V, int64_t D, bool wbf16, const ColMap &m, int *ni
     const int nparts = dense_parts(V, D);
     if (m.vec != 4 || m.npanels != 1 || nparts > kMaxClusterCtas)
         return false;
-    const int R1 = (16 / m.cpt) < 1 ? 1 : (16 / m.cpt);
+    const int R1 = reduce_rows_per_thread(V, D, m);
     const int rows_per_it = (kThreads / m.tpr) * R1;
     const int64_t rows = (V + nparts - 1) / nparts;
     const int64_t n = (rows + rows_per_it - 1) / rows_per_it;
     const size_t slots = (size_t)n * R1 * m.cpt * kThreads;
-    const size_t bytes = slots * (16 + (wbf16 ? 8 : 16)) + (size_t)4 * D * sizeof(float) +
+    // kept G and W, then D floats each of the column partial, the old c and
+    // the new c, rg x D floats of row-group sums, and the group sums of c
+    const size_t bytes = slots * (16 + (wbf16 ? 8 : 16)) +
+                         (size_t)(3 + kThreads / m.tpr) * D * sizeof(float) +
                          (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float);
     if (bytes > kSmallSmemMax)
         return false;
@@ -793,8 +807,8 @@ k_dense_cluster(SmallArgs a)
     F *keepG = reinterpret_cast<F *>(sm_dyn);
     WT *keepW = reinterpret_cast<WT *>(sm_dyn + nslot * 16);
     float *cpart = reinterpret_cast<float *>(sm_dyn + nslot * (16 + sizeof(WT)));
-    float *comb = cpart + a.D;
-    float *cold = comb + a.D;
+    float *comb = cpart + a.D;  // (256 / tpr) x D floats
+    float *cold = comb + (size_t)(kThreads / a.tpr) * a.D;
     float *cnew = cold + a.D;
     float *csum_sh = cnew + a.D;
     __shared__ float rsum_own;
@@ -1114,21 +1128,7 @@ k_rowonly_dense(void *__restrict__ W, const float *__restrict__ G, float *__rest
         }
     } else {
         float *colsh = reinterpret_cast<float *>(ro_dyn + (ASYNC ? rowonly_stage_bytes<CPT, R, BF16>() : 0));
-        for (int q = 0; q < rg; ++q) {
-            if (g == q) {
-#pragma unroll
-                for (int c = 0; c < CPT; ++c) {
-                    const int col = l + c * tpr;
-                    if (col < DV)
-#pragma unroll
-                        for (int e = 0; e < VEC; ++e)
-                            colsh[col * VEC + e] = (q == 0) ? acc[c][e] : colsh[col * VEC + e] + acc[c][e];
-                }
-            }
-            __syncthreads();
-        }
-        for (int j = tid; j < D; j += kThreads)
-            out[j] = colsh[j];
+        combine_row_groups<VEC, CPT>(acc, colsh, out, D, DV, tpr, rg, g, l);  // rg x D floats
     }
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
@@ -1180,10 +1180,10 @@ __global__ void k_shard_pack(const float *__restrict__ colpart, const float *__r
     }
 }
 
-template <int VEC, int CPT>
+// R1: rows per thread of the reduce pass, reduce_rows_per_thread(V, D, map)
+template <int VEC, int CPT, int R1>
 cudaError_t launch_dense_t(const DenseArgs &a)
 {
-    constexpr int R1 = (16 / CPT) < 1 ? 1 : (16 / CPT);
     constexpr int R3 = (8 / CPT) < 1 ? 1 : (8 / CPT);
     const int nparts = dense_parts(a.V, a.D);
     const int D = (int)a.D;
@@ -1199,7 +1199,7 @@ cudaError_t launch_dense_t(const DenseArgs &a)
     const int pw = a.map.pw;
     const int ld = (int)a.D;
     auto cols = [&](int q) { return (q + 1 < np) ? pw : (int)(a.D - (int64_t)q * pw); };
-    const size_t shmem = (rg > 1) ? (size_t)pw * sizeof(float) : 0;
+    const size_t shmem = (rg > 1) ? (size_t)rg * pw * sizeof(float) : 0;  // the row groups' column sums
 
     // With tracing, events sit between the kernels and each launch simply
     // follows the previous one; without, kernels 2 and 3 use programmatic
@@ -1295,6 +1295,8 @@ cudaError_t launch_dense_t(const DenseArgs &a)
             // G and W in shared memory
             auto *k = a.wbf16 ? k_dense_cluster<CPT, R1, true> : k_dense_cluster<CPT, R1, false>;
             e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+            if (e == cudaSuccess && nparts > 8)
+                e = cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
             if (e != cudaSuccess)
                 return e;
             SmallArgs sa{a.W, a.G, a.r, a.c, sc, a.V, D, a.map.tpr, nits, kc, a.eps, a.lr_signed, a.variant};
@@ -1440,18 +1442,20 @@ bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m)
 cudaError_t launch_dense_step(const DenseArgs &a)
 {
     if (a.map.vec == 4) {
+        const bool half = reduce_rows_per_thread(a.V, a.D, a.map) == 8;
         switch (a.map.cpt) {
-        case 1: return launch_dense_t<4, 1>(a);
-        case 2: return launch_dense_t<4, 2>(a);
-        case 4: return launch_dense_t<4, 4>(a);
-        case 8: return launch_dense_t<4, 8>(a);
+        case 1: return half ? launch_dense_t<4, 1, 8>(a) : launch_dense_t<4, 1, 16>(a);
+        case 2: return launch_dense_t<4, 2, 8>(a);
+        case 4: return launch_dense_t<4, 4, 4>(a);
+        case 8: return launch_dense_t<4, 8, 2>(a);
         }
     } else {
+        const bool half = reduce_rows_per_thread(a.V, a.D, a.map) == 8;
         switch (a.map.cpt) {
-        case 1: return launch_dense_t<1, 1>(a);
-        case 2: return launch_dense_t<1, 2>(a);
-        case 4: return launch_dense_t<1, 4>(a);
-        case 8: return launch_dense_t<1, 8>(a);
+        case 1: return half ? launch_dense_t<1, 1, 8>(a) : launch_dense_t<1, 1, 16>(a);
+        case 2: return launch_dense_t<1, 2, 8>(a);
+        case 4: return launch_dense_t<1, 4, 4>(a);
+        case 8: return launch_dense_t<1, 8, 2>(a);
         }
     }
     return cudaErrorInvalidValue;

@@ -108,7 +108,7 @@ bool choose_colmap(int64_t D, bool vec4_ok, ColMap *m);
 
 // Small tables run the whole dense step as one thread-block cluster launch
 // (see ember_dense.cu); the plan and the launch count of a dense step.
-constexpr int kMaxClusterCtas = 8;
+constexpr int kMaxClusterCtas = 16;  // a non-portable cluster size past 8
 constexpr size_t kSmallSmemMax = 200 << 10;
 bool small_table_plan(int64_t V, int64_t D, bool wbf16, const ColMap &m, int *nits, size_t *smem);
 int dense_step_launches(int64_t V, int64_t D, bool wbf16, int variant, bool vec4);
@@ -176,12 +176,12 @@ struct DenseArgs {
 };
 
 // CTAs of the dense step's reduce and apply grids for a V x D table: one
-// per kMinCtaElems elements of G (so that a table of up to 8 x 8192
-// elements has at most 8 CTAs and runs as one cluster launch), at most
+// per kMinCtaElems elements of G (so that a table of up to 16 x 4096
+// elements has at most 16 CTAs and can run as one cluster launch), at most
 // kGridCtas and at most one per row.  A function of (V, D) only, so the
 // per-CTA partial sums -- and the results -- are the same on every run and
 // device.
-constexpr int64_t kMinCtaElems = 8192;
+constexpr int64_t kMinCtaElems = 4096;
 inline int dense_parts(int64_t V, int64_t D)
 {
     int64_t n = (V * D + kMinCtaElems - 1) / kMinCtaElems;
@@ -190,6 +190,22 @@ inline int dense_parts(int64_t V, int64_t D)
     if (n > V)
         n = V;
     return (int)(n < 1 ? 1 : n);
+}
+
+// Rows a thread of the reduce pass takes per iteration (its rows in flight):
+// 16 / cpt, halved for rows of one access per thread when a CTA's rows fit
+// in half an iteration, so that on a small table every thread reduces (and,
+// in the one-launch step, updates) half as many rows.  A function of (V, D)
+// and the column map only, like the grid: every form of the step forms the
+// same per-CTA partials.
+inline int reduce_rows_per_thread(int64_t V, int64_t D, const ColMap &m)
+{
+    const int r = (16 / m.cpt) < 1 ? 1 : 16 / m.cpt;
+    if (m.cpt != 1)
+        return r;
+    const int nparts = dense_parts(V, D);
+    const int64_t rows = (V + nparts - 1) / nparts;
+    return rows <= (int64_t)(kThreads / m.tpr) * (r / 2) ? r / 2 : r;
 }
 
 // Default limit of a bounded wait inside a kernel (grid barriers, mbarrier

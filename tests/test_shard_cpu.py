@@ -24,9 +24,9 @@ def built():
 
 
 def cta_rows(V, D):
-    """Row boundaries of the whole-table step's CTAs: one per 8192 elements
+    """Row boundaries of the whole-table step's CTAs: one per 4096 elements
     of G, at most 304 (two per SM of the GB300) and at most one per row."""
-    nparts = max(1, min(V, 304, -(-V * D // 8192)))
+    nparts = max(1, min(V, 304, -(-V * D // 4096)))
     return [b * V // nparts for b in range(nparts + 1)]
 
 
