@@ -110,7 +110,8 @@ __device__ __forceinline__ void reduce_rows(const float *__restrict__ G, float *
                                             int64_t V, int D, int ld, int tpr, const StepConsts &kc,
                                             float *__restrict__ G_stage, float *__restrict__ rowpart,
                                             RowSpan span, int cta,
-                                            float *__restrict__ comb, typename Vec<VEC>::F *__restrict__ keep)
+                                            float *__restrict__ comb, typename Vec<VEC>::F *__restrict__ keep,
+                                            float *__restrict__ keep_r = nullptr)
 {
     using F = typename Vec<VEC>::F;
     constexpr int kWarps = kThreads / 32;
@@ -219,6 +220,8 @@ __device__ __forceinline__ void reduce_rows(const float *__restrict__ G, float *
                     }
                     const float rn = ema_pair(kc.ema, r[i], sum * kc.inv_D);
                     r[i] = rn;
+                    if (keep_r)  // the one-launch step's update reads it back here
+                        keep_r[i - row0] = rn;
                     rsum += rn;
                 }
             }
@@ -747,7 +750,7 @@ struct SmallArgs {
 // (one 16- or 8-byte slot per thread, per row and access of each reduce
 // iteration), then D floats of the column partial, (256 / tpr) x D floats of
 // the row groups' sums, D floats each of the old c and the new c (then the
-// column scales), and ceil(D/32) floats.
+// column scales), ceil(D/32) floats, and the new r of the CTA's rows.
 template <int CPT, int R, bool BF16>
 __host__ __device__ constexpr size_t small_slots(int nits) { return (size_t)nits * R * CPT * kThreads; }
 
@@ -768,10 +771,11 @@ bool small_table_plan(int64_t V, int64_t D, bool wbf16, const ColMap &m, int *ni
     const int64_t n = (rows + rows_per_it - 1) / rows_per_it;
     const size_t slots = (size_t)n * R1 * m.cpt * kThreads;
     // kept G and W, then D floats each of the column partial, the old c and
-    // the new c, rg x D floats of row-group sums, and the group sums of c
+    // the new c, rg x D floats of row-group sums, the group sums of c and
+    // the new r of the CTA's rows
     const size_t bytes = slots * (16 + (wbf16 ? 8 : 16)) +
                          (size_t)(3 + kThreads / m.tpr) * D * sizeof(float) +
-                         (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float);
+                         (size_t)((D + kStateCols - 1) / kStateCols) * sizeof(float) + (size_t)rows * sizeof(float);
     if (bytes > kSmallSmemMax)
         return false;
     *nits = (int)n;
@@ -811,6 +815,7 @@ k_dense_cluster(SmallArgs a)
     float *cold = comb + (size_t)(kThreads / a.tpr) * a.D;
     float *cnew = cold + a.D;
     float *csum_sh = cnew + a.D;
+    float *rnew = csum_sh + (a.D + kStateCols - 1) / kStateCols;  // the new r of this CTA's rows
     __shared__ float rsum_own;
 
     const int D = a.D, DV = D / VEC, tid = threadIdx.x;
@@ -848,7 +853,7 @@ k_dense_cluster(SmallArgs a)
         cold[j] = a.c[j];
 
     reduce_rows<VEC, CPT, R, false, true>(a.G, a.r, cpart, &rsum_own, a.V, D, D, tpr, a.kc, nullptr, nullptr, span,
-                                          cta, comb, keepG);
+                                          cta, comb, keepG, rnew);
     cluster_barrier();  // every CTA's partials are in its shared memory
 
     // the column pass for every column, as column_group forms it
@@ -908,7 +913,7 @@ k_dense_cluster(SmallArgs a)
             const int64_t i = row0 + (int64_t)it * rows_per_it + (int64_t)g * R + k;
             if (i >= row1)
                 continue;
-            const float rs = (a.variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(__ldcg(a.r + i) * inv_bc);
+            const float rs = (a.variant == EMBER_VARIANT_COL) ? 1.f : sqrtf(rnew[i - row0] * inv_bc);
 #pragma unroll
             for (int c = 0; c < CPT; ++c) {
                 const int col = l + c * tpr;
