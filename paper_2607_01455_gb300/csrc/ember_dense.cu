@@ -469,8 +469,10 @@ __device__ float block_fx_total(Load load, int n)
     __shared__ unsigned long long ss[kStateWarps];
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
-    unsigned e = 0;
-    for (int b = threadIdx.x; b < n; b += kStateThreads)
+    // each thread's first value is loaded once and kept for the second pass
+    const float first = ((int)threadIdx.x < n) ? load(threadIdx.x) : 0.f;
+    unsigned e = fx_key(first);
+    for (int b = threadIdx.x + kStateThreads; b < n; b += kStateThreads)
         e = max(e, fx_key(load(b)));
     e = __reduce_max_sync(0xffffffffu, e);
     if (lane == 0)
@@ -480,8 +482,8 @@ __device__ float block_fx_total(Load load, int n)
 #pragma unroll
     for (int q = 0; q < kStateWarps; ++q)
         E = max(E, ek[q]);
-    unsigned long long s = 0;
-    for (int b = threadIdx.x; b < n; b += kStateThreads)
+    unsigned long long s = fx_of(first, E);  // 0 for a zero
+    for (int b = threadIdx.x + kStateThreads; b < n; b += kStateThreads)
         s += fx_of(load(b), E);
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
@@ -646,10 +648,13 @@ k_state_dense(ColSource src, float *__restrict__ rsum_part, int nrsum, float *__
     if (!am_last)
         return;
     __threadfence();
+    // this thread's first group sum of c, loaded together with the sums of r
+    const float c_first = ((int)threadIdx.x < ngroups) ? __ldcg(csum_part + threadIdx.x) : 0.f;
     const float r_total = (src.sums != nullptr)
                               ? fx_value(src.sums[D], src.scales[D])
                               : block_fx_total([&](int b) { return __ldcg(rsum_part + b); }, nrsum);
-    const Norm n = normaliser(r_total, [&](int q) { return __ldcg(csum_part + q); }, ngroups, kc);
+    const Norm n = normaliser(
+        r_total, [&](int q) { return q == (int)threadIdx.x ? c_first : __ldcg(csum_part + q); }, ngroups, kc);
     if (threadIdx.x == 0) {
         sc->s = n.s;
         sc->rbar = n.rbar;
