@@ -367,21 +367,35 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
     const int j = group * kStateCols + lane;
+    const float c_old = (w == 0 && j < D) ? __ldcg(c + j) : 0.f;  // loaded with the partials
     unsigned long long S = 0;
     unsigned E = 0;
     if (src.sums == nullptr && src.nparts <= kRegParts * kStateWarps) {
         // up to kRegParts partial rows per warp: one trip to L2, the values
         // kept in registers for both the largest key and the sum
+        // (in chunks of 8, the chunks past this warp's last row skipped)
+        constexpr int kChunk = 8;
+        const int kv = (src.nparts - w + kStateWarps - 1) / kStateWarps;  // this warp's rows
         float v[kRegParts];
         unsigned e = 0;
 #pragma unroll
-        for (int k = 0; k < kRegParts; ++k) {
-            const int b = w + k * kStateWarps;
-            v[k] = (b < src.nparts && j < D) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+        for (int k0 = 0; k0 < kRegParts; k0 += kChunk) {
+            if (k0 >= kv)
+                break;
+#pragma unroll
+            for (int k = k0; k < k0 + kChunk; ++k) {
+                const int b = w + k * kStateWarps;
+                v[k] = (b < src.nparts && j < D) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+            }
         }
 #pragma unroll
-        for (int k = 0; k < kRegParts; ++k)
-            e = max(e, fx_key(v[k]));
+        for (int k0 = 0; k0 < kRegParts; k0 += kChunk) {
+            if (k0 >= kv)
+                break;
+#pragma unroll
+            for (int k = k0; k < k0 + kChunk; ++k)
+                e = max(e, fx_key(v[k]));
+        }
         emax_sh[w][lane] = e;
         __syncthreads();
 #pragma unroll
@@ -389,8 +403,13 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
             E = max(E, emax_sh[q][lane]);
         unsigned long long s = 0;
 #pragma unroll
-        for (int k = 0; k < kRegParts; ++k)
-            s += fx_of(v[k], E);
+        for (int k0 = 0; k0 < kRegParts; k0 += kChunk) {
+            if (k0 >= kv)
+                break;
+#pragma unroll
+            for (int k = k0; k < k0 + kChunk; ++k)
+                s += fx_of(v[k], E);
+        }
         ssum_sh[w][lane] = s;
         __syncthreads();
         if (w == 0)
@@ -446,7 +465,7 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
         float cn = 0.f;
         if (j < D) {
             const float m = fx_value(S, E) * kc.inv_V;
-            cn = ema_pair(kc.ema, __ldcg(c + j), m);
+            cn = ema_pair(kc.ema, c_old, m);
             c[j] = cn;
         }
 #pragma unroll
