@@ -350,6 +350,10 @@ struct ColSource {
     int nparts;
     const unsigned long long *sums;       // nullptr, or [D] totals
     const unsigned char *scales;          // their scale exponents
+    // partial row b holds nonzero sums only in columns [s pcols, (s + 1) pcols)
+    // of slice s = b % pstride (the sparse step's segment-sum CTAs); pstride
+    // 1: every row covers every column
+    int pstride = 1, pcols = 0;
 };
 
 constexpr int kStateWarps = kStateThreads / 32;
@@ -368,14 +372,18 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
     const int w = threadIdx.x >> 5;
     const int j = group * kStateCols + lane;
     const float c_old = (w == 0 && j < D) ? __ldcg(c + j) : 0.f;  // loaded with the partials
+    // the partial rows of this group's slice: b = sigma + p pstride, p < np
+    // (the other rows are zero in these columns and add nothing)
+    const int sigma = (src.pstride > 1) ? (group * kStateCols) / src.pcols : 0;
+    const int np = (src.nparts - sigma + src.pstride - 1) / src.pstride;
     unsigned long long S = 0;
     unsigned E = 0;
-    if (src.sums == nullptr && src.nparts <= kRegParts * kStateWarps) {
+    if (src.sums == nullptr && np <= kRegParts * kStateWarps) {
         // up to kRegParts partial rows per warp: one trip to L2, the values
         // kept in registers for both the largest key and the sum
         // (in chunks of 8, the chunks past this warp's last row skipped)
         constexpr int kChunk = 8;
-        const int kv = (src.nparts - w + kStateWarps - 1) / kStateWarps;  // this warp's rows
+        const int kv = (np - w + kStateWarps - 1) / kStateWarps;  // this warp's rows
         float v[kRegParts];
         unsigned e = 0;
 #pragma unroll
@@ -384,8 +392,8 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
                 break;
 #pragma unroll
             for (int k = k0; k < k0 + kChunk; ++k) {
-                const int b = w + k * kStateWarps;
-                v[k] = (b < src.nparts && j < D) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+                const int p = w + k * kStateWarps;
+                v[k] = (p < np && j < D) ? __ldcg(src.colpart + (int64_t)(sigma + p * src.pstride) * D + j) : 0.f;
             }
         }
 #pragma unroll
@@ -421,12 +429,12 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
         // pass 1: the largest key of the column (loads batched for latency)
         unsigned e = 0;
         if (j < D)
-            for (int b0 = w; b0 < src.nparts; b0 += kBatch * kStateWarps) {
+            for (int p0 = w; p0 < np; p0 += kBatch * kStateWarps) {
                 float v[kBatch];
 #pragma unroll
                 for (int k = 0; k < kBatch; ++k) {
-                    const int b = b0 + k * kStateWarps;
-                    v[k] = (b < src.nparts) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+                    const int p = p0 + k * kStateWarps;
+                    v[k] = (p < np) ? __ldcg(src.colpart + (int64_t)(sigma + p * src.pstride) * D + j) : 0.f;
                 }
 #pragma unroll
                 for (int k = 0; k < kBatch; ++k)
@@ -440,12 +448,12 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
         // pass 2: the exact total (the partials are still in L2)
         unsigned long long s = 0;
         if (j < D)
-            for (int b0 = w; b0 < src.nparts; b0 += kBatch * kStateWarps) {
+            for (int p0 = w; p0 < np; p0 += kBatch * kStateWarps) {
                 float v[kBatch];
 #pragma unroll
                 for (int k = 0; k < kBatch; ++k) {
-                    const int b = b0 + k * kStateWarps;
-                    v[k] = (b < src.nparts) ? __ldcg(src.colpart + (int64_t)b * D + j) : 0.f;
+                    const int p = p0 + k * kStateWarps;
+                    v[k] = (p < np) ? __ldcg(src.colpart + (int64_t)(sigma + p * src.pstride) * D + j) : 0.f;
                 }
 #pragma unroll
                 for (int k = 0; k < kBatch; ++k)
@@ -1430,11 +1438,11 @@ cudaError_t launch_dense_t(const DenseArgs &a)
 cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
                          float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &kc,
                          cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
-                         int nslices, int nrow_ctas, const int32_t *uniq, int rsum_base)
+                         int nslices, int nrow_ctas, const int32_t *uniq, int rsum_base, int pstride, int pcols)
 {
     const int ngroups = (D + kStateCols - 1) / kStateCols;
     RowPass rp{r_rows, slot, rowpart, nslices, nrow_ctas, uniq, rsum_base};
-    const ColSource src{colpart, nparts, nullptr, nullptr};
+    const ColSource src{colpart, nparts, nullptr, nullptr, pstride, pcols};
     return launch_k(k_state_dense, dim3(ngroups + nrow_ctas), dim3(kStateThreads), 0, stream, pdl, src,
                     rsum_part, nrsum, c, csum_part, sc, V, D, kc, rp);
 }

@@ -266,7 +266,8 @@ inline StepConsts make_consts(double beta2, double one_minus_beta2, int64_t V, i
 cudaError_t launch_state(const float *colpart, int nparts, float *rsum_part, int nrsum, float *c,
                          float *csum_part, DevScalars *sc, int64_t V, int D, const StepConsts &k,
                          cudaStream_t stream, bool pdl, float *r_rows, int32_t *slot, const float *rowpart,
-                         int nslices, int nrow_ctas, const int32_t *uniq = nullptr, int rsum_base = 0);
+                         int nslices, int nrow_ctas, const int32_t *uniq = nullptr, int rsum_base = 0,
+                         int pstride = 1, int pcols = 0);
 
 struct SparseArgs {
     int64_t V, D, N;

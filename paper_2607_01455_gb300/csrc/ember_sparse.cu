@@ -933,8 +933,9 @@ cudaError_t launch_sparse_t(const SparseArgs &a)
     // sums of r follow the segment-sum CTAs' sums of the decayed rows
     const int64_t ub = (a.N + kStateThreads - 1) / kStateThreads;
     const int GU = (int)(ub < kRsumParts - G ? ub : kRsumParts - G);
+    // (segment-sum CTA b writes only the columns of its slice b % NS)
     launch_state(colpart, G, rsum_part, G + GU, a.c, csum_part, sc, a.V, D, kc, a.stream, tr.pdl(), a.r, slot, rowpart,
-                 NS, GU, uniq, G);
+                 NS, GU, uniq, G, NS, kThreads * VEC);
     tr.mark();
     // one launch per column panel (one unless D is wider than a CTA's row)
     const int np = a.map.npanels, pw = a.map.pw;
