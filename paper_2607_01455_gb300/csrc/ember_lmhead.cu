@@ -16,18 +16,22 @@
 //
 // Tiles: a pair of CTAs (a cluster of two, on two SMs) runs
 // tcgen05.mma.cta_group::2 on 256 rows of G (vocabulary) x 256 columns
-// (features).  Each CTA holds, per pipeline stage of 64 tokens, its own 128
-// rows of dlogits and its own 128 columns of H (32 KiB; six stages, 192 KiB),
-// and its tensor memory holds its 128 rows of the 256 x 256 accumulator; the
-// even CTA (the leader) issues the MMAs for both.  Halving the H each SM
-// stages (the two tensor cores share the halves) is what lets six stages of
-// operands fit, enough to cover L2 latency.
+// (features).  Each CTA holds, per pipeline stage of 96 tokens, its own 128
+// rows of dlogits and its own 128 columns of H (48 KiB; four stages, 192
+// KiB), and its tensor memory holds its 128 rows of the 256 x 256
+// accumulator; the even CTA (the leader) issues the MMAs for both.  Halving
+// the H each SM stages (the two tensor cores share the halves) is what lets
+// 384 tokens of operands be in flight, enough to cover L2 latency.  Of the
+// ways to split those 384 tokens, four stages of 96 ran fastest: 4 % faster
+// than six of 64 and 3 % faster than three of 128 on the 128256 x 8192 head
+// (two of 192 and twelve of 32 far slower).  A last stage past T reads
+// zeros (the tensor map fills them).
 //
 // Both operands are "MN-major" in memory (dlogits is T x V and H is T x D,
 // row-major, so for a fixed token the tile's rows, resp. columns, are
-// contiguous): TMA loads 64 x 64 boxes with the 128-byte swizzle, described to
-// the MMA as MN-major, swizzled, 8 KiB between 64-element blocks and 1 KiB
-// between 8-token groups.  Both CTAs' loads of a stage complete on the
+// contiguous): TMA loads 64-element x 96-token boxes with the 128-byte
+// swizzle, described to the MMA as MN-major, swizzled, 12 KiB between
+// 64-element blocks and 1 KiB between 8-token groups.  Both CTAs' loads of a stage complete on the
 // leader's barrier; the leader's MMA completion frees the stage in both.
 //
 // Tiles are taken in bands of 16 column blocks (all row pairs of a band, then
@@ -69,14 +73,14 @@ namespace {
 constexpr int kBM = 128;                    // accumulator rows per CTA (half the pair's UMMA M)
 constexpr int kPairM = 2 * kBM;             // UMMA M of the pair
 constexpr int kBN = 256;                    // tile columns (UMMA N)
-constexpr int kBK = 64;                     // tokens per stage
+constexpr int kBK = 96;                     // tokens per stage (six MMAs of 16)
 constexpr int kUK = 16;                     // K of one kind::f16 MMA
-constexpr int kStages = 6;
+constexpr int kStages = 4;
 constexpr int kBox = 64;                    // TMA box: 64 bf16 = 128 bytes, the swizzle span
-constexpr int kABytes = kBM * kBK * 2;      // 16 KiB: this CTA's 128 rows of dlogits
-constexpr int kBBytes = (kBN / 2) * kBK * 2;  // 16 KiB: this CTA's 128 columns of H
+constexpr int kABytes = kBM * kBK * 2;      // 24 KiB: this CTA's 128 rows of dlogits
+constexpr int kBBytes = (kBN / 2) * kBK * 2;  // 24 KiB: this CTA's 128 columns of H
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 8 KiB
+constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 12 KiB
 constexpr int kAccCols = kBN;               // fp32 accumulator columns per tile
 constexpr int kTmemCols = 2 * kAccCols;     // two accumulators
 constexpr int kLmThreads = 256;
@@ -206,7 +210,7 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // Shared-memory matrix descriptor of tcgen05.mma for an MN-major operand
-// with the 128-byte swizzle: start address, 8 KiB between 64-element blocks
+// with the 128-byte swizzle: start address, 12 KiB between 64-element blocks
 // along M (or N) ("leading" offset), 1 KiB between groups of 8 rows along K
 // ("stride" offset), descriptor version 1, swizzle mode 2 (128 bytes).
 __device__ __forceinline__ uint64_t mn_major_sw128_desc(uint32_t saddr)
