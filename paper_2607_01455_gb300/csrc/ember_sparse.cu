@@ -266,14 +266,20 @@ k_sp_segments(const uint64_t *__restrict__ sorted, int64_t N, int64_t V,
     __shared__ int sh[kSortThreads / 32];
     grid_dep_wait();  // per-tile counts
     grid_dep_launch();
-    if (threadIdx.x == 0) {
+    {
+        // run heads and valid ids of the tiles before this one: a thread per
+        // tile, then the block's sums (one trip to L2, not one per tile)
         int a = 0, b = 0;
-        for (int t = 0; t < (int)blockIdx.x; ++t) {
+        for (int t = threadIdx.x; t < (int)blockIdx.x; t += kSortThreads) {
             a += tilecnt[2 * t];
             b += tilecnt[2 * t + 1];
         }
-        pre[0] = a;
-        pre[1] = b;
+        a = block_sum_int(a, sh);
+        b = block_sum_int(b, sh);
+        if (threadIdx.x == 0) {
+            pre[0] = a;
+            pre[1] = b;
+        }
     }
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
     const int64_t p0 = (int64_t)blockIdx.x * kSortTile + (int64_t)threadIdx.x * kKeysPerThread;
