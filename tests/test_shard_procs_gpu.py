@@ -64,7 +64,7 @@ def _rank(rank, port, out):
                 else:
                     ref.step_dense(Wref, G, 1e-3, t)
                 Gs = {k: G[r0:r0 + n].contiguous() for k, (r0, n) in plan.items()}
-                # round 1: the largest exponent per column, all-reduced with MAX
+                # first exchange: the largest exponent per column, all-reduced with MAX
                 scales = torch.zeros(D + 1, dtype=torch.uint8, device=dev)
                 for k in mine:
                     sk = torch.zeros(D + 1, dtype=torch.uint8, device=dev)
@@ -73,7 +73,7 @@ def _rank(rank, port, out):
                 scales_h = scales.cpu()
                 dist.all_reduce(scales_h, op=dist.ReduceOp.MAX)
                 scales = scales_h.to(dev)
-                # round 2: the fixed-point totals, all-reduced with SUM
+                # second exchange: the fixed-point totals, all-reduced with SUM
                 sums = torch.zeros(D + 1, dtype=torch.int64, device=dev)
                 for k in mine:
                     pk = torch.zeros(D + 1, dtype=torch.int64, device=dev)
