@@ -16,21 +16,22 @@
 //
 // Tiles: a pair of CTAs (a cluster of two, on two SMs) runs
 // tcgen05.mma.cta_group::2 on 256 rows of G (vocabulary) x 256 columns
-// (features).  Each CTA holds, per pipeline stage of 96 tokens, its own 128
-// rows of dlogits and its own 128 columns of H (48 KiB; four stages, 192
+// (features).  Each CTA holds, per pipeline stage of 80 tokens, its own 128
+// rows of dlogits and its own 128 columns of H (40 KiB; five stages, 200
 // KiB), and its tensor memory holds its 128 rows of the 256 x 256
 // accumulator; the even CTA (the leader) issues the MMAs for both.  Halving
 // the H each SM stages (the two tensor cores share the halves) is what lets
-// 384 tokens of operands be in flight, enough to cover L2 latency.  Of the
-// ways to split those 384 tokens, four stages of 96 ran fastest: 4 % faster
-// than six of 64 and 3 % faster than three of 128 on the 128256 x 8192 head
-// (two of 192 and twelve of 32 far slower).  A last stage past T reads
-// zeros (the tensor map fills them).
+// 400 tokens of operands be in flight, enough to cover L2 latency.  How they
+// are split matters: on the 128256 x 8192 head four stages of 96 ran 4 %
+// faster than six of 64 and 3 % faster than three of 128 (two of 192 and
+// twelve of 32 far slower), and five of 80, with one G staging block per
+// epilogue warp instead of two to make room, 1 % faster again.  A last
+// stage past T reads zeros (the tensor map fills them).
 //
 // Both operands are "MN-major" in memory (dlogits is T x V and H is T x D,
 // row-major, so for a fixed token the tile's rows, resp. columns, are
-// contiguous): TMA loads 64-element x 96-token boxes with the 128-byte
-// swizzle, described to the MMA as MN-major, swizzled, 12 KiB between
+// contiguous): TMA loads 64-element x 80-token boxes with the 128-byte
+// swizzle, described to the MMA as MN-major, swizzled, 10 KiB between
 // 64-element blocks and 1 KiB between 8-token groups.  Both CTAs' loads of a stage complete on the
 // leader's barrier; the leader's MMA completion frees the stage in both.
 //
@@ -73,14 +74,14 @@ namespace {
 constexpr int kBM = 128;                    // accumulator rows per CTA (half the pair's UMMA M)
 constexpr int kPairM = 2 * kBM;             // UMMA M of the pair
 constexpr int kBN = 256;                    // tile columns (UMMA N)
-constexpr int kBK = 96;                     // tokens per stage (six MMAs of 16)
+constexpr int kBK = 80;                     // tokens per stage (five MMAs of 16)
 constexpr int kUK = 16;                     // K of one kind::f16 MMA
-constexpr int kStages = 4;
+constexpr int kStages = 5;
 constexpr int kBox = 64;                    // TMA box: 64 bf16 = 128 bytes, the swizzle span
-constexpr int kABytes = kBM * kBK * 2;      // 24 KiB: this CTA's 128 rows of dlogits
-constexpr int kBBytes = (kBN / 2) * kBK * 2;  // 24 KiB: this CTA's 128 columns of H
+constexpr int kABytes = kBM * kBK * 2;      // 20 KiB: this CTA's 128 rows of dlogits
+constexpr int kBBytes = (kBN / 2) * kBK * 2;  // 20 KiB: this CTA's 128 columns of H
 constexpr int kStageBytes = kABytes + kBBytes;
-constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 12 KiB
+constexpr int kBlockBytes = kBox * kBK * 2; // one 64-wide box: 10 KiB
 constexpr int kAccCols = kBN;               // fp32 accumulator columns per tile
 constexpr int kTmemCols = 2 * kAccCols;     // two accumulators
 constexpr int kLmThreads = 256;
@@ -100,10 +101,11 @@ struct LmSmemTail {
     int abort;
     float xch[2][4][32];       // per-warp column sums, double-buffered
 };
-// Epilogue staging of G for the TMA store: per epilogue warp, two 32 x 32
-// fp32 blocks (4 KiB each, 128-byte swizzled rows).
+// Epilogue staging of G for the TMA store: per epilogue warp, kStoreBufs
+// 32 x 32 fp32 blocks (4 KiB each, 128-byte swizzled rows).
+constexpr int kStoreBufs = 1;
 constexpr int kStoreBlockBytes = 32 * 32 * 4;
-constexpr int kStoreBytes = 4 * 2 * kStoreBlockBytes;
+constexpr int kStoreBytes = 4 * kStoreBufs * kStoreBlockBytes;
 constexpr size_t kLmSmemBytes = 1024 + (size_t)kStages * kStageBytes + kStoreBytes + sizeof(LmSmemTail);
 static_assert(kLmSmemBytes <= 232448, "over the 227 KiB of shared memory a CTA may use");
 
@@ -210,7 +212,7 @@ __device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence:
 __device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // Shared-memory matrix descriptor of tcgen05.mma for an MN-major operand
-// with the 128-byte swizzle: start address, 12 KiB between 64-element blocks
+// with the 128-byte swizzle: start address, 10 KiB between 64-element blocks
 // along M (or N) ("leading" offset), 1 KiB between groups of 8 rows along K
 // ("stride" offset), descriptor version 1, swizzle mode 2 (128 bytes).
 __device__ __forceinline__ uint64_t mn_major_sw128_desc(uint32_t saddr)
@@ -538,7 +540,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
         uint32_t acc_phase = 0;
         int buf = 0;
         int sbuf = 0;
-        unsigned char *my_stage = gstage + (size_t)q * 2 * kStoreBlockBytes;
+        unsigned char *my_stage = gstage + (size_t)q * kStoreBufs * kStoreBlockBytes;
         const uint64_t pol_g = l2_policy(2);
         for (int gt = gt0; gt < npair_tiles; gt += gstep) {
             int mb, nb;
@@ -563,7 +565,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                 // swizzle order; then one TMA store, clipped at V and D
                 if (row0 < V) {
                     if (lane == 0)
-                        tma_store_wait_read<1>();  // this staging block's previous store has read it
+                        tma_store_wait_read<kStoreBufs - 1>();  // this staging block's previous store has read it
                     __syncwarp();
                     unsigned char *blk = my_stage + sbuf * kStoreBlockBytes + lane * 128;
 #pragma unroll
@@ -574,7 +576,7 @@ k_lmhead_grad(const __grid_constant__ CUtensorMap tm_dl, const __grid_constant__
                     __syncwarp();
                     if (lane == 0)
                         tma_store_2d(&tm_g, smem_addr(my_stage + sbuf * kStoreBlockBytes), col0, row0, pol_g);
-                    sbuf ^= 1;
+                    sbuf = (sbuf + 1 == kStoreBufs) ? 0 : sbuf + 1;
                 }
 #pragma unroll
                 for (int e = 0; e < 32; ++e) {
