@@ -489,17 +489,18 @@ __device__ __forceinline__ void column_group(const ColSource &src, int group, fl
 // whole CTA of kStateThreads threads; every thread gets the result.  The
 // loader reads global memory through L2 (the values were written by other
 // CTAs) or another CTA's shared memory in a cluster.
-template <typename Load>
+template <int NT = kStateThreads, typename Load>
 __device__ float block_fx_total(Load load, int n)
 {
-    __shared__ unsigned ek[kStateWarps];
-    __shared__ unsigned long long ss[kStateWarps];
+    constexpr int kNW = NT / 32;  // warps
+    __shared__ unsigned ek[kNW];
+    __shared__ unsigned long long ss[kNW];
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
     // each thread's first value is loaded once and kept for the second pass
     const float first = ((int)threadIdx.x < n) ? load(threadIdx.x) : 0.f;
     unsigned e = fx_key(first);
-    for (int b = threadIdx.x + kStateThreads; b < n; b += kStateThreads)
+    for (int b = threadIdx.x + NT; b < n; b += NT)
         e = max(e, fx_key(load(b)));
     e = __reduce_max_sync(0xffffffffu, e);
     if (lane == 0)
@@ -507,10 +508,10 @@ __device__ float block_fx_total(Load load, int n)
     __syncthreads();
     unsigned E = 0;
 #pragma unroll
-    for (int q = 0; q < kStateWarps; ++q)
+    for (int q = 0; q < kNW; ++q)
         E = max(E, ek[q]);
     unsigned long long s = fx_of(first, E);  // 0 for a zero
-    for (int b = threadIdx.x + kStateThreads; b < n; b += kStateThreads)
+    for (int b = threadIdx.x + NT; b < n; b += NT)
         s += fx_of(load(b), E);
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
@@ -520,28 +521,31 @@ __device__ float block_fx_total(Load load, int n)
     __syncthreads();
     unsigned long long S = 0;
 #pragma unroll
-    for (int q = 0; q < kStateWarps; ++q)
+    for (int q = 0; q < kNW; ++q)
         S += ss[q];
     __syncthreads();
     return fx_value(S, E);
 }
 
 // The normaliser from the total of r (r_total, over the whole table) and the
-// per-group sums of the new c (load(q), q < ngroups), by a whole CTA; every
-// thread gets it.  The group sums are added in a fixed order (thread t takes
-// groups t, t + 256, ... in order, then a fixed butterfly, then the warps in
-// order), so every CTA that runs this forms the same bits.
+// per-group sums of the new c (load(q), q < ngroups), by a whole CTA of NT
+// threads; every thread gets it.  The group sums are added in a fixed order
+// (thread t takes groups t, t + NT, ... in order, then a fixed butterfly,
+// then the warps in order), so every CTA that runs this forms the same bits,
+// and for up to 256 groups CTAs of 256 and 512 threads form the same sums
+// (each thread holds at most one group; the extra warps add zeros).
 struct Norm {
     float s, rbar, cbar, inv_s;
 };
-template <typename Load>
+template <int NT = kStateThreads, typename Load>
 __device__ Norm normaliser(float r_total, Load load, int ngroups, const StepConsts &kc)
 {
-    __shared__ float part[kStateWarps];
+    constexpr int kNW = NT / 32;  // warps
+    __shared__ float part[kNW];
     const int lane = threadIdx.x & 31;
     const int w = threadIdx.x >> 5;
     float csum = 0.f;
-    for (int q = threadIdx.x; q < ngroups; q += kStateThreads)
+    for (int q = threadIdx.x; q < ngroups; q += NT)
         csum += load(q);
 #pragma unroll
     for (int o = 16; o >= 1; o >>= 1)
@@ -550,7 +554,7 @@ __device__ Norm normaliser(float r_total, Load load, int ngroups, const StepCons
         part[w] = csum;
     __syncthreads();
     csum = 0.f;
-    for (int q = 0; q < kStateWarps; ++q)
+    for (int q = 0; q < kNW; ++q)
         csum += part[q];
     __syncthreads();
     Norm n;
@@ -891,7 +895,7 @@ k_dense_cluster(SmallArgs a)
     // the column pass for every column, as column_group forms it
     const int lane = tid & 31, w = tid >> 5;
     const int ngroups = (D + kStateCols - 1) / kStateCols;
-    for (int q = w; q < ngroups; q += kStateWarps) {
+    for (int q = w; q < ngroups; q += kThreads / 32) {
         const int j = q * kStateCols + lane;
         float v[kMaxClusterCtas];
         unsigned E = 0;
@@ -916,9 +920,9 @@ k_dense_cluster(SmallArgs a)
         if (lane == 0)
             csum_sh[q] = cn;
     }
-    const float r_total = block_fx_total([&](int b) { return ld_dsmem(&rsum_own, b); }, (int)nb);
+    const float r_total = block_fx_total<kThreads>([&](int b) { return ld_dsmem(&rsum_own, b); }, (int)nb);
     cluster_arrive();  // done reading the other CTAs' shared memory
-    const Norm n = normaliser(r_total, [&](int q) { return csum_sh[q]; }, ngroups, a.kc);
+    const Norm n = normaliser<kThreads>(r_total, [&](int q) { return csum_sh[q]; }, ngroups, a.kc);
     if (cta == 0) {
         for (int j = tid; j < D; j += kThreads)
             a.c[j] = cnew[j];

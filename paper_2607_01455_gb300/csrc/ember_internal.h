@@ -24,13 +24,14 @@ constexpr int kSparseCtasPerSm = 3;
 constexpr int kSparseCtas = kSms * kSparseCtasPerSm;
 constexpr int kPartRows = kSparseCtas > kGridCtas ? kSparseCtas : kGridCtas;
 
-// The state pass reduces 32 columns per CTA.  Its row pass runs up to
-// kMaxRowCtas CTAs: about one row per thread for the LM-head step (whose
+// The state pass reduces 32 columns per CTA of kStateThreads threads (16
+// warps, so that each warp adds few per-CTA partial rows).  Its row pass runs
+// up to kMaxRowCtas CTAs: about one row per thread for the LM-head step (whose
 // rows each sum ceil(D/256) slices) and for a dense step in column panels
 // (one slice per panel), and kRowBatch rows per thread for the sparse step
 // (whose untouched rows only decay).
 constexpr int kStateCols = 32;
-constexpr int kStateThreads = 256;
+constexpr int kStateThreads = 512;
 constexpr int kMaxRowCtas = 1024;
 constexpr int kRowBatch = 8;
 constexpr int kRsumParts = kMaxRowCtas > kGridCtas ? kMaxRowCtas : kGridCtas;
